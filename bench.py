@@ -1,0 +1,355 @@
+"""Benchmark of the routed-expert step: MoE-layer decode tokens/s at batch 1.
+
+Workload (default): 4 MoE layers, hidden 2048, 64 experts, top-8, intermediate 768, Q8_0,
+256 decode tokens at batch 1 per step, Zipf(1.1) routing with 0.6 reuse of the previous
+token's set, expert cache 35% of each layer's experts (22 slots).  A step is the whole
+256-token sequence through all 4 layers from a cold cache; `value` = tokens / s where a token
+passes all 4 layers.  Inputs (activations, planted router bias, router weights) are resident
+in HBM, the split-pack is in pinned host memory, misses are materialised inside the step.
+
+Each step is one CUDA graph replay of the 1024 C-ABI calls (captured once); L2 is flushed
+(a 512 MB write) between steps, outside the per-step CUDA events.  The kernel breakdown comes
+from CUDA events the library records around every launch, on the launching stream; they are
+captured into the graph, so they time the launches of the timed replays themselves.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--cache-pct P] [--impl mawforge|reference]
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = "l4e64"
+N_TOKENS = 256
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index, self.proc = index, None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+                self.lines = [l for l in out.splitlines() if l.strip()]
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            f = [v.strip() for v in line.split(",")]
+            if len(f) < 7:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx = float(f[1])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[3:7]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def build_workload(torch, mf, synth, cache_pct, device):
+    cfg = synth.CONFIGS[WORKLOAD]
+    L, H, E, k, I, q = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    model = mf.Model(L, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(cache_pct, 1 << 62, 0, 0, 1, 0))
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    buf = np.empty(plan.payload_bytes, np.uint8)
+    for l in range(L):
+        for e in range(E):
+            synth.payload(cfg.model_seed, l, e, H, I, q, out=buf)
+            mf.mf_pack_put(ctx, l, e, buf)
+    route = cfg.route_classes[0]
+    x = np.stack([synth.activations(0, l, 0, 0, N_TOKENS, H) for l in range(L)], 1)  # [T, L, H]
+    bias = np.stack([synth.plant_bias(synth.routes(0, l, 0, E, k, N_TOKENS, route.zipf_s, route.reuse), E)
+                     for l in range(L)], 1)  # [T, L, E]
+    wr = torch.from_numpy(np.stack([synth.router_weights(cfg.model_seed, l, E, H) for l in range(L)])).to(device)
+    return cfg, model, plan, ctx, x, bias, wr
+
+
+def run_mawforge(args):
+    import torch
+    import paper_2607_09686_gb300 as mf
+    import synth
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    cfg, model, plan, ctx, x_np, bias_np, wr = build_workload(torch, mf, synth, args.cache_pct, device)
+    L, H, E, k = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k
+    x = torch.from_numpy(x_np).to(device)
+    bias = torch.from_numpy(bias_np).to(device)
+    y = torch.empty(N_TOKENS, L, H, device=device)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=device)
+    stream = torch.cuda.Stream(device)
+
+    def step_calls():
+        mf.mf_reset(ctx, 0, stream)
+        for t in range(N_TOKENS):
+            for l in range(L):
+                mf.mf_moe_forward(ctx, l, x[t, l], wr[l], bias[t, l], 1, y[t, l], None, None, stream)
+
+    # one graph per step (the 1024 calls of a 256-token sequence), captured through the C ABI with
+    # the library's per-kernel event records inside, so the kernel times come from the timed replays
+    mf.mf_timing(ctx, True)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        step_calls()  # untimed eager pass: warms the pool
+        stream.synchronize()
+        mf.mf_timing(ctx, True)
+        with torch.cuda.graph(graph, stream=stream):
+            step_calls()
+    torch.cuda.synchronize()
+
+    def one_step(ev0, ev1):
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            ev0.record(stream)
+            graph.replay()
+            ev1.record(stream)
+
+    for _ in range(args.warmup):
+        one_step(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+    torch.cuda.synchronize()
+
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    kt = {name: [0.0, 0] for name in mf.KERNEL_CLASSES}
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            one_step(*evs[i])
+            for name, (kms, n) in mf.mf_timing_read(ctx).items():  # waits for this replay (outside its events)
+                kt[name][0] += kms
+                kt[name][1] += n
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    step_ms = [a.elapsed_time(b) for a, b in evs]
+    ms = sum(step_ms) / len(step_ms)
+    if ws > 1:
+        t = torch.tensor([ms], device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        torch.distributed.barrier()
+        ms = float(t.item())
+    st = mf.mf_stats(ctx, -1)  # every step starts cold (mf_reset), so these are one step's counters
+    mf.mf_timing(ctx, False)
+
+    # end to end through the host-buffer entry point: per token, pinned host x/bias in, y out
+    xh = torch.from_numpy(x_np).pin_memory()
+    bh = torch.from_numpy(bias_np).pin_memory()
+    yh = torch.empty(N_TOKENS, L, H).pin_memory()
+    e2e_graph = torch.cuda.CUDAGraph()
+
+    def e2e_calls():
+        mf.mf_reset(ctx, 0, stream)
+        for t in range(N_TOKENS):
+            for l in range(L):
+                mf.mf_moe_forward_host(ctx, l, xh[t, l], wr[l], bh[t, l], 1, yh[t, l], None, None, stream)
+
+    with torch.cuda.stream(stream):
+        e2e_calls()
+        stream.synchronize()
+        with torch.cuda.graph(e2e_graph, stream=stream):
+            e2e_calls()
+    torch.cuda.synchronize()
+    e2e_ms = []
+    for i in range(args.warmup + args.steps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            flush.zero_()
+            a.record(stream)
+            e2e_graph.replay()
+            b.record(stream)
+        b.synchronize()
+        if i >= args.warmup:
+            e2e_ms.append(a.elapsed_time(b))
+    y_dev = y.cpu()
+    assert torch.equal(y_dev, yh), "host-buffer path disagrees with the device path"
+
+    hbm, peak_kind = _peaks()
+    steps_per_tok = L
+    payload = plan.payload_bytes
+    # algorithmic bytes of one gate/up launch (k experts' gate+up blocks) and one down launch
+    gu_bytes = k * 2 * cfg.inter * (H // 32) * 34 + 4 * H + 4 * k * cfg.inter
+    dn_bytes = k * H * (cfg.inter // 32) * 34 + 4 * k * cfg.inter + 4 * H
+    ms_gu, n_gu = kt["gateup_swiglu"]
+    ms_dn, n_dn = kt["down_combine"]
+    ms_mat, n_mat = kt["materialize"]
+    gemv_gbs = (gu_bytes * n_gu + dn_bytes * n_dn) / ((ms_gu + ms_dn) * 1e-3) / 1e9
+    gu_gbs = gu_bytes / (ms_gu / n_gu * 1e-3) / 1e9
+    tokens = N_TOKENS * args.steps * ws
+    value = N_TOKENS / (ms * 1e-3) * ws
+    clocks = clk.summary()
+    kernels = {name: {"ms_total": round(v[0], 4), "launches": v[1],
+                      "us_per_launch": round(1e3 * v[0] / v[1], 3) if v[1] else None} for name, v in kt.items()}
+    line = {
+        "metric": "MoE-layer decode tokens/s at batch 1 (token = all 4 MoE layers)",
+        "value": round(value, 2),
+        "unit": "tokens/s",
+        "n_gpus": ws,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms, 4),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "q8_0 weights, f32 activations and accumulation",
+        "data": "synthetic (seeded; random-init Q8_0 experts; planted Zipf routing)",
+        "config": {"workload": f"{WORKLOAD}: 4 MoE layers, hidden 2048, 64 experts, top-8, inter 768, Q8_0, "
+                               f"256 decode tokens batch 1, Zipf 1.1 + 0.6 reuse, cache {args.cache_pct:g}%",
+                   "cache_pct": args.cache_pct, "slots_per_layer": plan.slots_per_layer,
+                   "tokens_per_step": N_TOKENS, "layers": L, "l2": "flushed between steps (512 MB write)",
+                   "execution": "one CUDA graph per step of the 1024 C-ABI calls"},
+        "cache": {"hit_rate": round(st["hits"] / max(1, st["accesses"]), 4),
+                  "materialized_bytes_per_token": st["bytes_materialized"] / N_TOKENS,
+                  "misses_per_token": st["misses"] / N_TOKENS, "accesses_per_step": st["accesses"]},
+        "roofline": {"bound": "hbm", "kernel": "gateup_swiglu (grouped dequant-GEMV, k experts' gate+up rows)",
+                     "achieved": round(gu_gbs, 1), "peak": hbm, "unit": "GB/s",
+                     "frac": round(gu_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": None,
+                     "gemv_pair_gbs": round(gemv_gbs, 1), "gemv_pair_frac": round(gemv_gbs / hbm, 4),
+                     "frac_of_8tbs": round(gemv_gbs / 8000.0, 4),
+                     "bytes_per_launch": {"gateup": gu_bytes, "down": dn_bytes}},
+        "kernels": kernels,
+        "copy": {"materialized_bytes_per_step": st["bytes_materialized"],
+                 "materialize_gbs": round(args.steps * st["bytes_materialized"] / (ms_mat * 1e-3) / 1e9, 1)
+                 if ms_mat else None},
+        "clocks": clocks,
+        "e2e": {"value": round(N_TOKENS / (statistics.mean(e2e_ms) * 1e-3) * ws, 2), "unit": "tokens/s",
+                "h2d_bytes_per_step": N_TOKENS * L * (H + E) * 4, "d2h_bytes_per_step": N_TOKENS * L * H * 4},
+        "gpu_launches": None,
+        "wall_s": round(wall, 3),
+    }
+    line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps  # + one reset kernel per step
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
+    mf.mf_destroy(ctx)
+    if rank == 0:
+        print(json.dumps(line))
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def cpu_baseline(n_tokens: int) -> dict:
+    """The CPU oracle, as it stands, on the first tokens of the same workload."""
+    import oracle
+    import synth
+    cfg = synth.CONFIGS[WORKLOAD]
+    L, H, E, k, I, q = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    route = cfg.route_classes[0]
+    pays = {}
+    lru = [oracle.LRU(E, int(np.floor(35.0 * E / 100 + 1e-9)), synth.payload_bytes(H, I, q)) for _ in range(L)]
+    xs = [synth.activations(0, l, 0, 0, n_tokens, H) for l in range(L)]
+    bs = [synth.plant_bias(synth.routes(0, l, 0, E, k, n_tokens, route.zipf_s, route.reuse), E) for l in range(L)]
+    wrs = [synth.router_weights(cfg.model_seed, l, E, H) for l in range(L)]
+    for l in range(L):  # payload generation is input preparation, outside the timing
+        for e in set(bs[l].nonzero()[1].tolist()):
+            pays[(l, e)] = synth.payload(cfg.model_seed, l, e, H, I, q)
+    t0 = time.perf_counter()
+    for t in range(n_tokens):
+        for l in range(L):
+            _, idx, _ = oracle.router(xs[l][t], wrs[l], bs[l][t], k)
+            lru[l].step(idx[None])
+            oracle.layer([pays.get((l, e)) for e in range(E)], q, H, I, k, wrs[l], bs[l][t:t + 1], xs[l][t:t + 1])
+    dt = time.perf_counter() - t0
+    cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return {"value": round(n_tokens / dt, 4), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"first {n_tokens} tokens of the same sequence, all {L} layers (router + LRU + fp64 layer)"}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    per_step = []
+    for i in range(args.warmup + args.steps):
+        r = cpu_baseline(args.cpu_tokens)
+        if i >= args.warmup:
+            per_step.append(r)
+    value = statistics.mean(r["value"] for r in per_step)
+    line = {"impl": "reference", "metric": "MoE-layer decode tokens/s at batch 1 (token = all 4 MoE layers)",
+            "value": round(value, 4), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * args.cpu_tokens / value, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64 (CPU oracle)", "data": "synthetic (seeded)",
+            "config": {"workload": f"{WORKLOAD} (the same workload; a bounded sample of it per step)",
+                       "tokens_per_step": args.cpu_tokens},
+            "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "kind": "oracle",
+                             "cores": per_step[0]["cores"], "sample": per_step[0]["sample"]},
+            "e2e": {"value": round(value, 4), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--cache-pct", type=float, default=35.0)
+    ap.add_argument("--impl", default="mawforge", choices=["mawforge", "reference"])
+    ap.add_argument("--cpu-tokens", type=int, default=16)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        import oracle
+        oracle.build()
+        run_reference(args)
+        return
+    import __graft_entry__
+    __graft_entry__.build()
+    run_mawforge(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,182 @@
+/*
+ * mawforge.h — C ABI of the routed-expert step of one MoE decoder layer on one GB300.
+ *
+ * Method: MawForge, "Memory-Bounded Expert Materialization for Local Mixture-of-Experts
+ * Inference" (arXiv 2607.09686).  Routed expert tensors live outside fast memory as
+ * per-layer, per-expert payloads (section "Split-Pack Representation"); a bounded set
+ * of per-layer slots holds the experts in use, and a miss copies the requested expert
+ * block into an available slot and updates the route-to-slot metadata (section
+ * "Native Serving Path"); a static check rejects a configuration whose lower bound
+ * L(p, n) = C + E(p) + K(n) exceeds the serving target before anything is loaded
+ * (section "Static Budget Check").
+ *
+ * Here the split-pack sits in pinned host memory, the slots in HBM, and one call of
+ * mf_moe_forward runs, for one layer and T tokens, entirely in CUDA kernels:
+ *   router logits + top-k + softmax over the chosen ->
+ *   slot resolve (per-layer LRU, hit / miss / eviction / byte counters) ->
+ *   materialisation of the missed payloads, pinned host -> HBM slot, on a side stream ->
+ *   dequantising gate/up projections + SwiGLU -> down projection + router-weighted combine.
+ *
+ * Conventions for every entry point:
+ *  - Return MF_OK (0) or a negative MF_E_* code; mf_strerror() names it.  A failing call
+ *    changes no state the caller can observe, except MF_E_CUDA after a kernel launch
+ *    failed (the context should then be destroyed).
+ *  - Pointers documented "device" must be device memory of the context's GPU (or
+ *    memory the GPU can address); "host" pointers are CPU memory.  The caller owns every
+ *    buffer it passes; the library owns the pinned pack, the HBM slot pool, its scratch,
+ *    its side stream and its events.
+ *  - A context is not thread-safe: one host thread at a time per context.
+ *  - Quantised weights use the GGUF block formats: Q8_0 = {binary16 d; int8 q[32]}
+ *    (34 B, w = d*q); Q4_0 = {binary16 d; uint8 qs[16]} (18 B, byte j holds element j
+ *    in its low nibble and element j+16 in its high nibble, w = d*(n-8)).
+ */
+#ifndef MAWFORGE_H
+#define MAWFORGE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---- */
+#define MF_OK 0
+#define MF_E_INVAL (-1)  /* an argument is out of range, NULL where required, or inconsistent */
+#define MF_E_BUDGET (-2) /* the static plan rejected this configuration */
+#define MF_E_OOM (-3)    /* pinned host or device allocation failed */
+#define MF_E_CUDA (-4)   /* a CUDA runtime call or kernel launch failed */
+#define MF_E_STATE (-5)  /* the call is not valid in the context's current state */
+
+/* ---- quantisation types (GGUF type ids) ---- */
+#define MF_Q4_0 2
+#define MF_Q8_0 8
+
+/* Shape of the routed-expert part of a model.  Each expert is a SwiGLU FFN with separate
+ * gate [inter x hidden], up [inter x hidden] and down [hidden x inter] tensors.
+ * Requirements: hidden and inter multiples of 32; 1 <= top_k <= 8; top_k <= n_experts <= 1024. */
+typedef struct mf_model {
+  int32_t n_layers, hidden, n_experts, top_k, inter, qtype;
+} mf_model_t;
+
+/* Static-plan request (section "Static Budget Check").
+ * cache_pct: expert-cache size as a percentage p of the experts of each layer (0..100).
+ * budget_bytes: the serving target; common_bytes: resident common tensors C;
+ * kv_bytes: K(n); max_tokens: the largest T a single mf_moe_forward call will pass. */
+typedef struct mf_plan_req {
+  double cache_pct;
+  uint64_t budget_bytes, common_bytes, kv_bytes;
+  int32_t max_tokens, reserved;
+} mf_plan_req_t;
+
+/* Static-plan result.
+ * slots_per_layer S = max(top_k, floor(p * n_experts / 100)), at most n_experts;
+ * payload_bytes: canonical GGUF bytes of one expert (gate + up + down);
+ * pool_bytes E(p) = n_layers * S * payload_bytes;
+ * lower_bound_bytes L = C + E(p) + K; accepted = (L <= budget);
+ * overhead_bytes O: this library's device scratch and slot-table bytes for max_tokens;
+ * footprint_bytes F = L + O (section "Static Budget Check"). */
+typedef struct mf_plan {
+  int32_t accepted, slots_per_layer;
+  uint64_t payload_bytes, pool_bytes, lower_bound_bytes, overhead_bytes, footprint_bytes;
+  int32_t max_tokens, reserved;
+} mf_plan_t;
+
+/* Cache counters of one layer, or summed over layers (section "Native Serving Path";
+ * the CLI of the paper reports hit rate and materialised expert bytes).
+ * accesses = hits + misses; bytes_materialized = misses * payload_bytes. */
+typedef struct mf_stats {
+  uint64_t accesses, hits, misses, evictions, bytes_materialized;
+} mf_stats_t;
+
+typedef struct mf_ctx mf_ctx_t;
+
+/* Canonical GGUF bytes of one expert payload.  Host only. */
+int mf_payload_bytes(const mf_model_t* model, uint64_t* out);
+
+/* Static budget check (section "Static Budget Check").  Host-only arithmetic, no GPU
+ * needed.  Fills *out even when rejecting; returns MF_E_BUDGET if L > budget. */
+int mf_plan(const mf_model_t* model, const mf_plan_req_t* req, mf_plan_t* out);
+
+/* Create a context on CUDA device `device`: allocates the pinned host pack
+ * (n_layers * n_experts payloads), the HBM slot pool (n_layers * S payloads), the slot
+ * table and the scratch for plan->max_tokens.  Refuses a rejected plan (MF_E_BUDGET).
+ * The pack is empty: fill it with mf_pack_put before the first mf_moe_forward. */
+int mf_create(mf_ctx_t** out, const mf_model_t* model, const mf_plan_t* plan, int device);
+
+/* Copy one expert's canonical GGUF payload (host memory, `bytes` must equal
+ * payload_bytes) into the pinned pack, repacked so quantised codes and scales are
+ * 16-byte aligned (the same bytes, regrouped; accounting stays at payload_bytes).
+ * The caller may free `payload` when the call returns.  Host only, synchronous; calls for
+ * distinct (layer, expert) pairs may run concurrently from several host threads. */
+int mf_pack_put(mf_ctx_t* ctx, int layer, int expert, const void* payload, uint64_t bytes);
+
+/* mf_create followed by mf_pack_put of payloads[layer * n_experts + expert] (host
+ * pointers, each payload_bytes long) for every layer and expert. */
+int mf_load_pack(mf_ctx_t** out, const mf_model_t* model, const mf_plan_t* plan,
+                 const void* const* payloads, int device);
+
+/* One routed-expert step of layer `layer` for T tokens, stream-ordered on `stream`
+ * (a cudaStream_t; NULL = the legacy default stream).
+ *   x          device float [T][hidden]      token activations
+ *   router_w   device float [n_experts][hidden]  router weights W_r
+ *   logit_bias device float [T][n_experts] or NULL, added to the logits in fp32
+ *   y          device float [T][hidden]      output: sum_j g_j * FFN_{e_j}(x_t)
+ *   idx_out    device int32 [T][top_k] or NULL: chosen experts, largest logit first
+ *              (ties to the lower expert id)
+ *   w_out      device float [T][top_k] or NULL: softmax of the chosen logits
+ * Each layer's cache is one LRU over that layer's calls, in call order: calls for one
+ * layer must be issued in token order.  Within a call the accesses are the distinct
+ * experts of the T tokens in (token, rank) first-occurrence order; when there are more
+ * than S of them they are processed in waves of S.  0 <= T <= plan max_tokens; T = 0
+ * does nothing.  Inputs must be finite.  Returns after enqueueing (no host sync). */
+int mf_moe_forward(mf_ctx_t* ctx, int layer, const float* x, const float* router_w,
+                   const float* logit_bias, int T, float* y, int32_t* idx_out, float* w_out,
+                   void* stream);
+
+/* As mf_moe_forward, with x, logit_bias, y, idx_out and w_out in HOST memory (pinned
+ * memory lets the copies overlap; pageable memory works but serialises).  Stages x and
+ * the bias into the context's device buffers, runs the step and copies the outputs back,
+ * all on `stream`.  The host buffers must stay valid until the stream reaches the end of
+ * the call (synchronise before reading y). */
+int mf_moe_forward_host(mf_ctx_t* ctx, int layer, const float* x, const float* router_w,
+                        const float* logit_bias, int T, float* y, int32_t* idx_out, float* w_out,
+                        void* stream);
+
+/* Cache counters of `layer`, or summed over all layers when layer = -1.  Synchronises
+ * the context's device work first.  reset != 0 zeroes the counters read. */
+int mf_stats(mf_ctx_t* ctx, int layer, mf_stats_t* out, int reset);
+
+/* Make every layer's cache cold and zero all counters; if slots_per_layer > 0, also set
+ * the number of slots in use per layer (top_k <= slots_per_layer <= the planned S).
+ * Stream-ordered on `stream`. */
+int mf_reset(mf_ctx_t* ctx, int slots_per_layer, void* stream);
+
+/* The access record of the most recent mf_moe_forward call of `layer`: for each access
+ * u < *n, the expert, its slot after the access and whether it hit.  Host arrays of
+ * `cap` entries; synchronises the context's device work first. */
+int mf_trace(mf_ctx_t* ctx, int layer, int32_t* experts, int32_t* slots, uint8_t* hits, int cap,
+             int* n);
+
+/* Per-kernel timing with CUDA events recorded on the stream each kernel runs on.
+ * enable != 0 starts recording (clearing earlier records); mf_timing_read synchronises,
+ * and writes for each kernel class (0 router, 1 resolve, 2 materialise, 3 gate/up+SwiGLU,
+ * 4 down+combine, 5 prefill grouped GEMM) the summed milliseconds and the number of launches
+ * into ms[6] and launches[6].  Calls captured into a CUDA graph while timing is on capture
+ * their event records as graph nodes; after each replay mf_timing_read reports that replay. */
+int mf_timing(mf_ctx_t* ctx, int enable);
+int mf_timing_read(mf_ctx_t* ctx, double* ms, int64_t* launches);
+
+/* Release everything the context owns (synchronises its streams first). NULL is a no-op. */
+void mf_destroy(mf_ctx_t* ctx);
+
+/* Static string naming a status code. */
+const char* mf_strerror(int status);
+
+/* Text of the last CUDA error seen by this library in the calling thread ("" if none). */
+const char* mf_last_cuda_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MAWFORGE_H */

@@ -1,0 +1,325 @@
+// Decode expert FFN: grouped dequantising GEMV over the experts resident in HBM slots.
+//
+//   h[t,j][r] = silu(sum_c Wg_e[r,c] x_t[c]) * sum_c Wu_e[r,c] x_t[c]     (gate/up + SwiGLU)
+//   y[t][c]   = sum_j g[t,j] * sum_r Wd_e[c,r] h[t,j][r]                  (down + combine)
+// with e = the expert routed at (t, j), W = d * q (Q8_0) or d * (n - 8) (Q4_0), silu(v) =
+// v / (1 + e^-v) (SwiGLU expert FFN with separate gate, up and down tensors, section
+// "Native Serving Path").  fp32 accumulation throughout.
+//
+// One warp per weight row.  Each lane holds whole 16-byte vectors of the row's codes in
+// registers (Q8_0: 16 weights, Q4_0: one 32-weight block) and reuses them for every token
+// the expert serves.  Codes are turned into floats exactly by placing each byte (or
+// nibble) in the low mantissa bits of 2^23 with a byte permute and subtracting 2^23 plus
+// the code offset (the int8 -> float "magic number" conversion of Kim et al., "Who says
+// elephants can't run", 2022), which costs one PRMT and one FADD per weight instead of an
+// integer-to-float conversion.  The scale multiplies each vector's partial dot product.
+// Cross-lane sums use a fixed xor-shuffle tree, so results are deterministic.
+#include "mf_internal.cuh"
+
+namespace mf {
+namespace {
+
+constexpr int kQ8 = MF_Q8_0;
+constexpr int kQ4 = MF_Q4_0;
+
+// four signed int8 codes of w dotted with x[0..3]
+__device__ __forceinline__ float dot4_q8(uint32_t w, float4 x, float acc) {
+  const uint32_t u = w ^ 0x80808080u;  // code + 128 in each byte
+  const float f0 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7540)) - 8388736.0f;  // 2^23 + 128
+  const float f1 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7541)) - 8388736.0f;
+  const float f2 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7542)) - 8388736.0f;
+  const float f3 = __uint_as_float(__byte_perm(u, 0x4B000000u, 0x7543)) - 8388736.0f;
+  acc = fmaf(f0, x.x, acc);
+  acc = fmaf(f1, x.y, acc);
+  acc = fmaf(f2, x.z, acc);
+  acc = fmaf(f3, x.w, acc);
+  return acc;
+}
+
+// four 4-bit codes (one per byte, already masked) dotted with x[0..3]; weight = n - 8
+__device__ __forceinline__ float dot4_q4(uint32_t n, float4 x, float acc) {
+  const float f0 = __uint_as_float(__byte_perm(n, 0x4B000000u, 0x7540)) - 8388616.0f;  // 2^23 + 8
+  const float f1 = __uint_as_float(__byte_perm(n, 0x4B000000u, 0x7541)) - 8388616.0f;
+  const float f2 = __uint_as_float(__byte_perm(n, 0x4B000000u, 0x7542)) - 8388616.0f;
+  const float f3 = __uint_as_float(__byte_perm(n, 0x4B000000u, 0x7543)) - 8388616.0f;
+  acc = fmaf(f0, x.x, acc);
+  acc = fmaf(f1, x.y, acc);
+  acc = fmaf(f2, x.z, acc);
+  acc = fmaf(f3, x.w, acc);
+  return acc;
+}
+
+// weights covered by one 16-byte vector
+template <int QT>
+struct Vec {
+  static constexpr int kW = QT == kQ8 ? 16 : 32;
+};
+
+// x values of vector v: Q8_0 16 contiguous floats; Q4_0 the 32 floats of block v
+template <int QT>
+struct XV {
+  float4 a[Vec<QT>::kW / 4];
+};
+
+template <int QT>
+__device__ __forceinline__ XV<QT> load_x(const float* __restrict__ xv) {
+  XV<QT> r;
+#pragma unroll
+  for (int i = 0; i < Vec<QT>::kW / 4; ++i) r.a[i] = __ldg(reinterpret_cast<const float4*>(xv) + i);
+  return r;
+}
+
+// unscaled dot product of one code vector with its x values
+template <int QT>
+__device__ __forceinline__ float dot_vec(uint4 w, const XV<QT>& x) {
+  float acc = 0.f;
+  if constexpr (QT == kQ8) {
+    acc = dot4_q8(w.x, x.a[0], acc);
+    acc = dot4_q8(w.y, x.a[1], acc);
+    acc = dot4_q8(w.z, x.a[2], acc);
+    acc = dot4_q8(w.w, x.a[3], acc);
+  } else {
+    // byte j: element j (low nibble), element j + 16 (high nibble)
+    const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      acc = dot4_q4(ws[i] & 0x0F0F0F0Fu, x.a[i], acc);
+      acc = dot4_q4((ws[i] >> 4) & 0x0F0F0F0Fu, x.a[4 + i], acc);
+    }
+  }
+  return acc;
+}
+
+template <int QT>
+__device__ __forceinline__ int scale_index(int v) {
+  return QT == kQ8 ? (v >> 1) : v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+  return v;
+}
+
+__device__ __forceinline__ const uint8_t* slot_base(const Dev& d, int layer, int slot) {
+  return d.pool + ((size_t)layer * d.S_alloc + slot) * d.lay.stride;
+}
+
+// ---------------------------------------------------------------- gate/up + SwiGLU
+// grid (ceil(I / 8), wave width); block 256 = 8 warps = 8 rows of gate and up.
+template <int QT, int VPL>
+__global__ void __launch_bounds__(256) k_gateup(Dev d, int layer, int wave, const float* __restrict__ x) {
+  const int u = wave * d.S_active + blockIdx.y;
+  if (u >= d.info[0]) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * 8 + warp;
+  if (r >= d.I) return;
+  const uint8_t* slot = slot_base(d, layer, d.uslot[u]);
+  const uint8_t* gq = slot + d.lay.gq + (size_t)r * d.lay.qrow_gu;
+  const uint8_t* uq = slot + d.lay.uq + (size_t)r * d.lay.qrow_gu;
+  const __half* gd = reinterpret_cast<const __half*>(slot + d.lay.gd) + (size_t)r * d.lay.nb_gu;
+  const __half* ud = reinterpret_cast<const __half*>(slot + d.lay.ud) + (size_t)r * d.lay.nb_gu;
+  const int nvec = d.lay.qrow_gu / 16;
+
+  uint4 wg[VPL], wu[VPL];
+  float sg[VPL], su[VPL];
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) {
+    const int v = lane + 32 * i;
+    if (v < nvec) {
+      wg[i] = ld_stream(gq + 16 * v);
+      wu[i] = ld_stream(uq + 16 * v);
+      sg[i] = __half2float(gd[scale_index<QT>(v)]);
+      su[i] = __half2float(ud[scale_index<QT>(v)]);
+    }
+  }
+  const int a0 = d.asg_off[u], a1 = d.asg_off[u + 1];
+  for (int a = a0; a < a1; ++a) {
+    const int pos = d.asg[a];
+    const float* xt = x + (size_t)(pos / d.k) * d.H;
+    float ag = 0.f, au = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) {
+      const int v = lane + 32 * i;
+      if (v < nvec) {
+        const XV<QT> xv = load_x<QT>(xt + v * Vec<QT>::kW);
+        ag = fmaf(dot_vec<QT>(wg[i], xv), sg[i], ag);
+        au = fmaf(dot_vec<QT>(wu[i], xv), su[i], au);
+      }
+    }
+    ag = warp_sum(ag);
+    au = warp_sum(au);
+    if (lane == 0) d.h[(size_t)pos * d.I + r] = ag / (1.0f + expf(-ag)) * au;
+  }
+}
+
+// ---------------------------------------------------------------- down + combine, one token
+// grid ceil(H / 8); block 256 = 8 warps = 8 output rows; JB experts' rows held at once.
+template <int QT, int VPL, int JB>
+__global__ void __launch_bounds__(256) k_down_single(Dev d, int layer, float* __restrict__ y) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x * 8 + warp;
+  if (c >= d.H) return;
+  const int k = d.k, nvec = d.lay.qrow_d / 16;
+  float acc = 0.f;
+  for (int j0 = 0; j0 < k; j0 += JB) {
+    uint4 w[JB][VPL];
+    float sc[JB][VPL];
+#pragma unroll
+    for (int jj = 0; jj < JB; ++jj) {
+      const int j = j0 + jj;
+      if (j < k) {
+        const uint8_t* slot = slot_base(d, layer, d.pos_slot[j]);
+        const uint8_t* q = slot + d.lay.dq + (size_t)c * d.lay.qrow_d;
+        const __half* s = reinterpret_cast<const __half*>(slot + d.lay.dd) + (size_t)c * d.lay.nb_d;
+#pragma unroll
+        for (int i = 0; i < VPL; ++i) {
+          const int v = lane + 32 * i;
+          if (v < nvec) {
+            w[jj][i] = ld_stream(q + 16 * v);
+            sc[jj][i] = __half2float(s[scale_index<QT>(v)]);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int jj = 0; jj < JB; ++jj) {
+      const int j = j0 + jj;
+      if (j < k) {
+        const float* hj = d.h + (size_t)j * d.I;
+        float part = 0.f;
+#pragma unroll
+        for (int i = 0; i < VPL; ++i) {
+          const int v = lane + 32 * i;
+          if (v < nvec) part = fmaf(dot_vec<QT>(w[jj][i], load_x<QT>(hj + v * Vec<QT>::kW)), sc[jj][i], part);
+        }
+        acc = fmaf(d.g[j], part, acc);
+      }
+    }
+  }
+  acc = warp_sum(acc);
+  if (lane == 0) y[c] = acc;
+}
+
+// ---------------------------------------------------------------- down, per assignment (T > 1)
+// grid (ceil(H / 8), wave width): part[t*k+j][c] = sum_r Wd[c,r] h[t*k+j][r]
+template <int QT, int VPL>
+__global__ void __launch_bounds__(256) k_down_partial(Dev d, int layer, int wave) {
+  const int u = wave * d.S_active + blockIdx.y;
+  if (u >= d.info[0]) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int c = blockIdx.x * 8 + warp;
+  if (c >= d.H) return;
+  const uint8_t* slot = slot_base(d, layer, d.uslot[u]);
+  const uint8_t* q = slot + d.lay.dq + (size_t)c * d.lay.qrow_d;
+  const __half* s = reinterpret_cast<const __half*>(slot + d.lay.dd) + (size_t)c * d.lay.nb_d;
+  const int nvec = d.lay.qrow_d / 16;
+  uint4 w[VPL];
+  float sc[VPL];
+#pragma unroll
+  for (int i = 0; i < VPL; ++i) {
+    const int v = lane + 32 * i;
+    if (v < nvec) {
+      w[i] = ld_stream(q + 16 * v);
+      sc[i] = __half2float(s[scale_index<QT>(v)]);
+    }
+  }
+  const int a0 = d.asg_off[u], a1 = d.asg_off[u + 1];
+  for (int a = a0; a < a1; ++a) {
+    const int pos = d.asg[a];
+    const float* hp = d.h + (size_t)pos * d.I;
+    float part = 0.f;
+#pragma unroll
+    for (int i = 0; i < VPL; ++i) {
+      const int v = lane + 32 * i;
+      if (v < nvec) part = fmaf(dot_vec<QT>(w[i], load_x<QT>(hp + v * Vec<QT>::kW)), sc[i], part);
+    }
+    part = warp_sum(part);
+    if (lane == 0) d.part[(size_t)pos * d.H + c] = part;
+  }
+}
+
+// y[t][c] = sum_j g[t,j] part[t*k+j][c], j in rank order
+__global__ void k_combine(Dev d, int T, float* __restrict__ y) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)T * d.H) return;
+  const int t = (int)(i / d.H), c = (int)(i % d.H);
+  float acc = 0.f;
+  for (int j = 0; j < d.k; ++j) acc = fmaf(d.g[t * d.k + j], d.part[((size_t)t * d.k + j) * d.H + c], acc);
+  y[i] = acc;
+}
+
+// smallest instantiated vectors-per-lane count covering `nvec` vectors
+int pick_vpl(int nvec) {
+  const int need = (nvec + 31) / 32;
+  if (need <= 1) return 1;
+  if (need <= 2) return 2;
+  if (need <= 3) return 3;
+  if (need <= 4) return 4;
+  if (need <= 6) return 6;
+  return 8;
+}
+
+template <int QT>
+cudaError_t gateup_q(const Dev& d, int layer, int wave, int width, const float* x, cudaStream_t s) {
+  dim3 grid((d.I + 7) / 8, width);
+  switch (pick_vpl(d.lay.qrow_gu / 16)) {
+    case 1: k_gateup<QT, 1><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+    case 2: k_gateup<QT, 2><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+    case 3: k_gateup<QT, 3><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+    case 4: k_gateup<QT, 4><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+    case 6: k_gateup<QT, 6><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+    default: k_gateup<QT, 8><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+  }
+  return cudaGetLastError();
+}
+
+template <int QT>
+cudaError_t down_single_q(const Dev& d, int layer, float* y, cudaStream_t s) {
+  dim3 grid((d.H + 7) / 8);
+  switch (pick_vpl(d.lay.qrow_d / 16)) {
+    case 1: k_down_single<QT, 1, 8><<<grid, 256, 0, s>>>(d, layer, y); break;
+    case 2: k_down_single<QT, 2, 8><<<grid, 256, 0, s>>>(d, layer, y); break;
+    case 3: k_down_single<QT, 3, 8><<<grid, 256, 0, s>>>(d, layer, y); break;
+    case 4: k_down_single<QT, 4, 4><<<grid, 256, 0, s>>>(d, layer, y); break;
+    case 6: k_down_single<QT, 6, 2><<<grid, 256, 0, s>>>(d, layer, y); break;
+    default: k_down_single<QT, 8, 2><<<grid, 256, 0, s>>>(d, layer, y); break;
+  }
+  return cudaGetLastError();
+}
+
+template <int QT>
+cudaError_t down_partial_q(const Dev& d, int layer, int wave, int width, cudaStream_t s) {
+  dim3 grid((d.H + 7) / 8, width);
+  switch (pick_vpl(d.lay.qrow_d / 16)) {
+    case 1: k_down_partial<QT, 1><<<grid, 256, 0, s>>>(d, layer, wave); break;
+    case 2: k_down_partial<QT, 2><<<grid, 256, 0, s>>>(d, layer, wave); break;
+    case 3: k_down_partial<QT, 3><<<grid, 256, 0, s>>>(d, layer, wave); break;
+    case 4: k_down_partial<QT, 4><<<grid, 256, 0, s>>>(d, layer, wave); break;
+    case 6: k_down_partial<QT, 6><<<grid, 256, 0, s>>>(d, layer, wave); break;
+    default: k_down_partial<QT, 8><<<grid, 256, 0, s>>>(d, layer, wave); break;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gateup(const Dev& d, int layer, int wave, int width, const float* x, cudaStream_t s) {
+  return d.qtype == kQ8 ? gateup_q<kQ8>(d, layer, wave, width, x, s) : gateup_q<kQ4>(d, layer, wave, width, x, s);
+}
+
+cudaError_t launch_down_single(const Dev& d, int layer, float* y, cudaStream_t s) {
+  return d.qtype == kQ8 ? down_single_q<kQ8>(d, layer, y, s) : down_single_q<kQ4>(d, layer, y, s);
+}
+
+cudaError_t launch_down_partial(const Dev& d, int layer, int wave, int width, cudaStream_t s) {
+  return d.qtype == kQ8 ? down_partial_q<kQ8>(d, layer, wave, width, s) : down_partial_q<kQ4>(d, layer, wave, width, s);
+}
+
+cudaError_t launch_combine(const Dev& d, int T, float* y, cudaStream_t s) {
+  const size_t n = (size_t)T * d.H;
+  k_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(d, T, y);
+  return cudaGetLastError();
+}
+
+}  // namespace mf

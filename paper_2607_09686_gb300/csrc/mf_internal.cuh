@@ -1,0 +1,121 @@
+// Internal declarations of the GB300 routed-expert library (not part of the C ABI).
+#pragma once
+
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "mawforge.h"
+
+namespace mf {
+
+constexpr int kMaxTopK = 8;
+constexpr int kMaxExperts = 1024;
+constexpr int kTimerClasses = 6;
+enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5 };
+
+// SoA layout of one expert slot, identical in the pinned pack and in the HBM pool.
+// Quantised codes of each tensor are contiguous row-major (Q8_0: 1 byte per weight,
+// Q4_0: the 16 code bytes of each block in GGUF order), scales are binary16 row-major
+// [rows][cols/32].  Every region starts on a 256-byte boundary.
+struct Layout {
+  uint64_t gq, uq, dq;  // byte offsets of the gate / up / down codes
+  uint64_t gd, ud, dd;  // byte offsets of the gate / up / down scales
+  uint64_t stride;      // bytes per slot (a multiple of 256)
+  uint64_t canonical;   // canonical GGUF payload bytes (what a miss accounts for)
+  int qrow_gu, qrow_d;  // code bytes per row: gate/up rows (hidden weights), down rows (inter weights)
+  int nb_gu, nb_d;      // 32-weight blocks per row
+};
+
+// Everything a kernel needs, passed by value.
+struct Dev {
+  // model
+  int L, H, E, k, I, qtype;
+  int S_alloc, S_active, T_max;
+  Layout lay;
+  // memory
+  const uint8_t* pack;  // pinned host pack [L][E] slots, device-addressable
+  uint8_t* pool;        // HBM slot pool [L][S_alloc] slots
+  // per-layer cache state
+  int32_t* slot_of;    // [L][E]        expert -> slot or -1
+  int32_t* expert_of;  // [L][S_alloc]  slot -> expert or -1
+  uint64_t* last_use;  // [L][S_alloc]  LRU time of the slot's last access
+  uint64_t* clock;     // [L]
+  uint64_t* stats;     // [L][5]        accesses, hits, misses, evictions, bytes
+  // trace of each layer's latest call
+  int32_t* tr_n;       // [L]
+  int32_t* tr_expert;  // [L][E]
+  int32_t* tr_slot;    // [L][E]
+  uint8_t* tr_hit;     // [L][E]
+  // per-call scratch
+  float* logits;       // [T_max][E]
+  unsigned* ticket;    // [T_max]       router last-block tickets (kept at zero between calls)
+  int32_t* idx;        // [T_max][k]
+  float* g;            // [T_max][k]
+  int32_t* uniq;       // [E]           distinct experts in access order
+  int32_t* uslot;      // [E]           their slots
+  int32_t* umiss;      // [E]           1 if the access missed
+  int32_t* asg_off;    // [E + 1]       assignments of unique expert u: asg[asg_off[u] .. asg_off[u+1])
+  int32_t* asg;        // [T_max * k]   assignment = t * k + j
+  int32_t* pos_slot;   // [T_max * k]   slot serving assignment t * k + j
+  int32_t* info;       // [2 + E]       U, number of waves, misses of wave w at 2 + w
+  int32_t* miss_list;  // [E + S_alloc] unique index of miss m of wave w at w * S_active + m
+  float* h;            // [T_max * k][I]  SwiGLU activations
+  float* part;         // [T_max * k][H]  per-assignment down outputs (T > 1)
+};
+
+// 16-byte streaming load that does not allocate in L1 (weights are read once per call)
+__device__ __forceinline__ uint4 ld_stream(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+
+}  // namespace mf
+
+struct mf_ctx {
+  mf_model_t model;
+  mf_plan_t plan;
+  int device;
+  mf::Dev d;
+  uint8_t* pack_host;      // cudaHostAlloc'ed pack (host pointer)
+  unsigned char* put_map;  // [L][E] which payloads have been put
+  int64_t n_put;
+  cudaStream_t side;       // materialisation stream
+  int max_waves;
+  cudaEvent_t* ev_fork;    // [max_waves + 1]
+  cudaEvent_t* ev_join;    // [max_waves + 1]
+  // staging for mf_moe_forward_host
+  float* stage_x;
+  float* stage_bias;
+  float* stage_y;
+  int32_t* stage_idx;
+  float* stage_w;
+  // event timing
+  int timing;
+  int timer_cap;
+  int timer_n[mf::kTimerClasses];
+  int64_t timer_dropped;
+  cudaEvent_t* timer_ev[mf::kTimerClasses];  // pairs: [2 * i], [2 * i + 1]
+  uint64_t overhead_bytes;
+};
+
+namespace mf {
+
+// layout of a slot for a model shape
+Layout make_layout(const mf_model_t& m);
+uint64_t canonical_payload_bytes(const mf_model_t& m);
+
+// kernel launchers (each returns the launch status)
+cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, cudaStream_t s);
+cudaError_t launch_resolve(const Dev& d, int layer, int T, cudaStream_t s);
+cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s);
+cudaError_t launch_gateup(const Dev& d, int layer, int wave, int wave_width, const float* x, cudaStream_t s);
+cudaError_t launch_down_single(const Dev& d, int layer, float* y, cudaStream_t s);
+cudaError_t launch_down_partial(const Dev& d, int layer, int wave, int wave_width, cudaStream_t s);
+cudaError_t launch_combine(const Dev& d, int T, float* y, cudaStream_t s);
+cudaError_t launch_reset(const Dev& d, cudaStream_t s);
+
+}  // namespace mf
