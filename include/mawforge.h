@@ -46,6 +46,7 @@ extern "C" {
 #define MF_E_OOM (-3)    /* pinned host or device allocation failed */
 #define MF_E_CUDA (-4)   /* a CUDA runtime call or kernel launch failed */
 #define MF_E_STATE (-5)  /* the call is not valid in the context's current state */
+#define MF_E_TIMEOUT (-6) /* a bounded wait inside a kernel gave up (reported by mf_check) */
 
 /* ---- quantisation types (GGUF type ids) ---- */
 #define MF_Q4_0 2
@@ -165,6 +166,12 @@ int mf_trace(mf_ctx_t* ctx, int layer, int32_t* experts, int32_t* slots, uint8_t
  * their event records as graph nodes; after each replay mf_timing_read reports that replay. */
 int mf_timing(mf_ctx_t* ctx, int enable);
 int mf_timing_read(mf_ctx_t* ctx, double* ms, int64_t* launches);
+
+/* Synchronise the device and report whether any kernel of this context gave up a bounded
+ * wait since the last check (MF_E_TIMEOUT; results of that call are then unreliable).
+ * Kernels never spin without a limit: a pipeline stage that is not filled or released
+ * within the limit makes the kernel record the failure and return. */
+int mf_check(mf_ctx_t* ctx);
 
 /* Release everything the context owns (synchronises its streams first). NULL is a no-op. */
 void mf_destroy(mf_ctx_t* ctx);

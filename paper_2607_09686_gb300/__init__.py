@@ -17,13 +17,13 @@ import os
 __all__ = [
     "MFError", "Model", "PlanReq", "Plan", "Stats", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
     "mf_payload_bytes", "mf_plan", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
-    "mf_moe_forward_host", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_destroy",
+    "mf_moe_forward_host", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_destroy",
     "mf_strerror", "mf_last_cuda_error",
 ]
 
 Q4_0 = 2
 Q8_0 = 8
-MF_OK, MF_E_INVAL, MF_E_BUDGET, MF_E_OOM, MF_E_CUDA, MF_E_STATE = 0, -1, -2, -3, -4, -5
+MF_OK, MF_E_INVAL, MF_E_BUDGET, MF_E_OOM, MF_E_CUDA, MF_E_STATE, MF_E_TIMEOUT = 0, -1, -2, -3, -4, -5, -6
 KERNEL_CLASSES = ("router", "resolve", "materialize", "gateup_swiglu", "down_combine", "prefill_gemm")
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmawforge.so")
@@ -75,6 +75,7 @@ _sig = {
     "mf_trace": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, ctypes.POINTER(_i32)]),
     "mf_timing": (_i32, [_vp, _i32]),
     "mf_timing_read": (_i32, [_vp, _vp, _vp]),
+    "mf_check": (_i32, [_vp]),
     "mf_destroy": (None, [_vp]),
     "mf_strerror": (ctypes.c_char_p, [_i32]),
     "mf_last_cuda_error": (ctypes.c_char_p, []),
@@ -205,6 +206,14 @@ def mf_timing_read(ctx: int) -> dict:
     n = (ctypes.c_int64 * 6)()
     _check(_lib.mf_timing_read(ctx, ms, n), "mf_timing_read")
     return {KERNEL_CLASSES[i]: (float(ms[i]), int(n[i])) for i in range(6)}
+
+
+def mf_check(ctx: int) -> int:
+    """0, or MF_E_TIMEOUT if a kernel of this context gave up a bounded wait (returned, not raised)."""
+    rc = _lib.mf_check(ctx)
+    if rc not in (MF_OK, MF_E_TIMEOUT):
+        _check(rc, "mf_check")
+    return rc
 
 
 def mf_destroy(ctx: int) -> None:

@@ -87,7 +87,7 @@ struct Carve {
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
   uint64_t logits, ticket, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
-  uint64_t sx, sb, sy, sidx, sw;
+  uint64_t work, err, sx, sb, sy, sidx, sw;
   uint64_t total;
 };
 
@@ -118,6 +118,8 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.miss_list = c.take<int32_t>(E + S);
   o.h = c.take<float>((uint64_t)Tm * k * I);
   o.part = c.take<float>(Tm > 1 ? (uint64_t)Tm * k * H : 1);
+  o.work = c.take<unsigned>(4);
+  o.err = c.take<unsigned>(1);
   o.sx = c.take<float>((uint64_t)Tm * H);
   o.sb = c.take<float>((uint64_t)Tm * E);
   o.sy = c.take<float>((uint64_t)Tm * H);
@@ -242,6 +244,7 @@ const char* mf_strerror(int status) {
     case MF_E_OOM: return "out of memory";
     case MF_E_CUDA: return "CUDA error";
     case MF_E_STATE: return "invalid state";
+    case MF_E_TIMEOUT: return "a bounded device-side wait gave up";
     default: return "unknown status";
   }
 }
@@ -361,6 +364,8 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.miss_list = reinterpret_cast<int32_t*>(base + so.miss_list);
   d.h = reinterpret_cast<float*>(base + so.h);
   d.part = reinterpret_cast<float*>(base + so.part);
+  d.work = reinterpret_cast<unsigned*>(base + so.work);
+  d.err = reinterpret_cast<unsigned*>(base + so.err);
   c->stage_x = reinterpret_cast<float*>(base + so.sx);
   c->stage_bias = reinterpret_cast<float*>(base + so.sb);
   c->stage_y = reinterpret_cast<float*>(base + so.sy);
@@ -399,6 +404,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
     free_ctx(c);
     return MF_E_INVAL;
   }
+  c->decode_pipe = decode_pipe_ok(d) && getenv("MF_DECODE_SIMPLE") == nullptr;
   *out = c;
   return MF_OK;
 }
@@ -453,11 +459,13 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   const int S = d.S_active;
 
   timer_mark(c, kTRouter, 0, s);
-  MF_CUDA(launch_router(d, x, router_w, logit_bias, T, s));
+  MF_CUDA(launch_router(d, x, router_w, logit_bias, T, layer, s));
   timer_mark(c, kTRouter, 1, s);
-  timer_mark(c, kTResolve, 0, s);
-  MF_CUDA(launch_resolve(d, layer, T, s));
-  timer_mark(c, kTResolve, 1, s);
+  if (T > 1) {  // one token per call: the router's last block resolved the slots already
+    timer_mark(c, kTResolve, 0, s);
+    MF_CUDA(launch_resolve(d, layer, T, s));
+    timer_mark(c, kTResolve, 1, s);
+  }
 
   long long accesses_max = (long long)T * d.k;
   if (accesses_max > d.E) accesses_max = d.E;
@@ -472,11 +480,17 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
     timer_mark(c, kTMaterialize, 1, c->side);
     MF_CUDA(cudaEventRecord(c->ev_join[w], c->side));
     MF_CUDA(cudaStreamWaitEvent(s, c->ev_join[w], 0));
+    const bool pipe = T == 1 && c->decode_pipe;
     timer_mark(c, kTGateUp, 0, s);
-    MF_CUDA(launch_gateup(d, layer, w, (int)width, x, s));
+    if (pipe)
+      MF_CUDA(launch_gateup_single(d, layer, x, s));
+    else
+      MF_CUDA(launch_gateup(d, layer, w, (int)width, x, s));
     timer_mark(c, kTGateUp, 1, s);
     timer_mark(c, kTDown, 0, s);
-    if (T == 1)
+    if (pipe)
+      MF_CUDA(launch_down_single_pipe(d, layer, y, s));
+    else if (T == 1)
       MF_CUDA(launch_down_single(d, layer, y, s));
     else
       MF_CUDA(launch_down_partial(d, layer, w, (int)width, s));
@@ -602,6 +616,20 @@ int mf_timing_read(mf_ctx_t* c, double* ms, int64_t* launches) {
     }
     ms[i] = acc;
     launches[i] = c->timer_n[i];
+  }
+  return MF_OK;
+}
+
+int mf_check(mf_ctx_t* c) {
+  if (!c) return MF_E_INVAL;
+  DevGuard guard(c->device);
+  if (!guard.ok) return cuda_fail(cudaSetDevice(c->device), "cudaSetDevice");
+  MF_CUDA(cudaDeviceSynchronize());
+  unsigned err = 0;
+  MF_CUDA(cudaMemcpy(&err, c->d.err, sizeof(err), cudaMemcpyDeviceToHost));
+  if (err) {
+    MF_CUDA(cudaMemset(c->d.err, 0, sizeof(unsigned)));
+    return MF_E_TIMEOUT;
   }
   return MF_OK;
 }

@@ -62,7 +62,50 @@ struct Dev {
   int32_t* miss_list;  // [E + S_alloc] unique index of miss m of wave w at w * S_active + m
   float* h;            // [T_max * k][I]  SwiGLU activations
   float* part;         // [T_max * k][H]  per-assignment down outputs (T > 1)
+  unsigned* work;      // [4]           work-queue counters of the pipelined decode kernels
+  unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
 };
+
+// ---- shared-memory pipeline primitives (mbarrier + bulk asynchronous copy, PTX ISA 8.x)
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity; false after `limit` polls (an error, never a
+// hang: the caller records it and stops using the pipeline).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit = (1u << 26)) {
+  for (uint32_t i = 0; i < limit; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+// bulk copy global -> this CTA's shared memory, completing `bytes` on the mbarrier
+// (addresses 16-byte aligned, bytes a multiple of 16)
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+__device__ __forceinline__ void named_bar_sync(int id, int threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
 
 // 16-byte streaming load that does not allocate in L1 (weights are read once per call)
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
@@ -100,6 +143,7 @@ struct mf_ctx {
   int64_t timer_dropped;
   cudaEvent_t* timer_ev[mf::kTimerClasses];  // pairs: [2 * i], [2 * i + 1]
   uint64_t overhead_bytes;
+  bool decode_pipe;  // batch-1 calls use the pipelined decode kernels
 };
 
 namespace mf {
@@ -109,7 +153,8 @@ Layout make_layout(const mf_model_t& m);
 uint64_t canonical_payload_bytes(const mf_model_t& m);
 
 // kernel launchers (each returns the launch status)
-cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, cudaStream_t s);
+cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
+                          cudaStream_t s);
 cudaError_t launch_resolve(const Dev& d, int layer, int T, cudaStream_t s);
 cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s);
 cudaError_t launch_gateup(const Dev& d, int layer, int wave, int wave_width, const float* x, cudaStream_t s);
@@ -117,5 +162,10 @@ cudaError_t launch_down_single(const Dev& d, int layer, float* y, cudaStream_t s
 cudaError_t launch_down_partial(const Dev& d, int layer, int wave, int wave_width, cudaStream_t s);
 cudaError_t launch_combine(const Dev& d, int T, float* y, cudaStream_t s);
 cudaError_t launch_reset(const Dev& d, cudaStream_t s);
+// batch-1 decode: pipelined gate/up + SwiGLU and down + combine (shared-memory bulk-copy stages)
+cudaError_t launch_gateup_single(const Dev& d, int layer, const float* x, cudaStream_t s);
+cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStream_t s);
+size_t decode_smem_bytes(const Dev& d, int which);
+bool decode_pipe_ok(const Dev& d);
 
 }  // namespace mf

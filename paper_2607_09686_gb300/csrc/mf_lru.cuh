@@ -1,0 +1,96 @@
+// Least-recently-used slot replacement of one layer, run by one warp (internal).
+//
+// Section "Native Serving Path": on a miss the runtime materialises the expert block into an
+// available slot and updates the route-to-slot metadata.  Accesses are processed one at a
+// time in order: a resident expert hits (its slot becomes the most recently used); otherwise
+// the lowest free slot is taken, or, with none free, the slot of the least recently used
+// expert, which is evicted.  Accesses are grouped in waves of S consecutive accesses; within a
+// wave no access evicts an expert accessed earlier in the same wave (those are the most recent
+// and fewer than S), so each wave's experts occupy distinct slots when the wave is computed.
+#pragma once
+
+#include "mf_internal.cuh"
+
+namespace mf {
+
+// State of the layer in shared memory: s_slot_of[E], s_expert_of[S_active], s_last[S_active].
+// Writes the call's access record (uniq, uslot, umiss, trace), per-wave miss lists and counts,
+// the counters and the clock.  All 32 lanes must call it; lane 0 does the writes.
+__device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const int* s_uniq, int* s_slot_of,
+                                         int* s_expert_of, uint64_t* s_last, int* s_uslot) {
+  const int lane = threadIdx.x & 31, E = d.E, S = d.S_active;
+  uint64_t clock = d.clock[layer];  // kept by lane 0
+  uint64_t hits = 0, misses = 0, evictions = 0;
+  int wave_miss = 0;
+  for (int u = 0; u < U; ++u) {
+    if (u % S == 0) wave_miss = 0;
+    const int e = s_uniq[u];
+    int s = s_slot_of[e];
+    const bool hit = s >= 0;
+    if (!hit) {
+      int found = -1;
+      for (int base = 0; base < S && found < 0; base += 32) {
+        const int q = base + lane;
+        const unsigned b = __ballot_sync(0xffffffffu, q < S && s_expert_of[q] < 0);
+        if (b) found = base + __ffs(b) - 1;
+      }
+      if (found < 0) {  // no free slot: evict the least recently used
+        uint64_t best = ~0ull;
+        int bq = 0x7fffffff;
+        for (int q = lane; q < S; q += 32)
+          if (s_last[q] < best) {
+            best = s_last[q];
+            bq = q;
+          }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) {
+          const uint64_t ob = __shfl_xor_sync(0xffffffffu, best, off);
+          const int oq = __shfl_xor_sync(0xffffffffu, bq, off);
+          if (ob < best || (ob == best && oq < bq)) {
+            best = ob;
+            bq = oq;
+          }
+        }
+        found = bq;
+        if (lane == 0) s_slot_of[s_expert_of[found]] = -1;
+        ++evictions;
+      }
+      s = found;
+      if (lane == 0) {
+        s_expert_of[s] = e;
+        s_slot_of[e] = s;
+        d.miss_list[(u / S) * S + wave_miss] = u;
+      }
+      ++wave_miss;
+      ++misses;
+    } else {
+      ++hits;
+    }
+    if (lane == 0) {
+      if (u % S == S - 1 || u == U - 1) d.info[2 + u / S] = wave_miss;
+      s_last[s] = ++clock;
+      s_uslot[u] = s;
+      d.uniq[u] = e;
+      d.uslot[u] = s;
+      d.umiss[u] = hit ? 0 : 1;
+      d.tr_expert[(size_t)layer * E + u] = e;
+      d.tr_slot[(size_t)layer * E + u] = s;
+      d.tr_hit[(size_t)layer * E + u] = hit ? 1 : 0;
+    }
+    __syncwarp();  // lane 0's shared-memory updates are seen by the whole warp at the next access
+  }
+  if (lane == 0) {
+    d.clock[layer] = clock;
+    uint64_t* st = d.stats + (size_t)layer * 5;
+    st[0] += (uint64_t)U;
+    st[1] += hits;
+    st[2] += misses;
+    st[3] += evictions;
+    st[4] += misses * d.lay.canonical;
+    d.info[0] = U;
+    d.info[1] = (U + S - 1) / S;
+    d.tr_n[layer] = U;
+  }
+}
+
+}  // namespace mf

@@ -5,16 +5,11 @@
 // One block per call.  Steps:
 //  1. the distinct experts of the call's T*k routes, in (token, rank) first-occurrence
 //     order, and for each the list of assignments t*k+j it serves;
-//  2. least-recently-used replacement over those accesses, one at a time (one warp):
-//     resident -> hit; otherwise the lowest free slot, or the slot of the least recently
-//     used expert, which is evicted;
-//  3. accesses grouped in waves of S consecutive accesses (S = slots in use).  Within a
-//     wave no access evicts an expert accessed earlier in the same wave (those are the
-//     most recent ones and fewer than S), so each wave's experts end up in distinct
-//     slots and the wave can be materialised and computed as one batch;
-//  4. counters (accesses, hits, misses, evictions, bytes = misses * payload) and the
+//  2. least-recently-used replacement over those accesses in waves of S (lru_warp);
+//  3. counters (accesses, hits, misses, evictions, bytes = misses * payload) and the
 //     access record of the call.
-#include "mf_internal.cuh"
+// With one token per call the router's last block does this itself (mf_router.cu).
+#include "mf_lru.cuh"
 
 namespace mf {
 namespace {
@@ -34,7 +29,7 @@ __global__ void __launch_bounds__(256) k_resolve(Dev d, int layer, int T) {
   __shared__ int s_U;
 
   const int tid = threadIdx.x, nt = blockDim.x;
-  const int warp = tid >> 5, lane = tid & 31;
+  const int warp = tid >> 5;
   int32_t* g_slot_of = d.slot_of + (size_t)layer * E;
   int32_t* g_expert_of = d.expert_of + (size_t)layer * d.S_alloc;
   uint64_t* g_last = d.last_use + (size_t)layer * d.S_alloc;
@@ -92,80 +87,7 @@ __global__ void __launch_bounds__(256) k_resolve(Dev d, int layer, int T) {
   }
 
   // LRU, one access at a time
-  if (warp == 0) {
-    uint64_t clock = d.clock[layer];  // kept by lane 0
-    uint64_t hits = 0, misses = 0, evictions = 0;
-    int wave_miss = 0;
-    for (int u = 0; u < U; ++u) {
-      if (u % S == 0) wave_miss = 0;
-      const int e = s_uniq[u];
-      int s = s_slot_of[e];
-      const bool hit = s >= 0;
-      if (!hit) {
-        int found = -1;
-        for (int base = 0; base < S && found < 0; base += 32) {
-          int q = base + lane;
-          unsigned b = __ballot_sync(0xffffffffu, q < S && s_expert_of[q] < 0);
-          if (b) found = base + __ffs(b) - 1;
-        }
-        if (found < 0) {
-          uint64_t best = ~0ull;
-          int bq = 0x7fffffff;
-          for (int q = lane; q < S; q += 32)
-            if (s_last[q] < best) {
-              best = s_last[q];
-              bq = q;
-            }
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) {
-            uint64_t ob = __shfl_xor_sync(0xffffffffu, best, off);
-            int oq = __shfl_xor_sync(0xffffffffu, bq, off);
-            if (ob < best || (ob == best && oq < bq)) {
-              best = ob;
-              bq = oq;
-            }
-          }
-          found = bq;
-          if (lane == 0) s_slot_of[s_expert_of[found]] = -1;
-          ++evictions;
-        }
-        s = found;
-        if (lane == 0) {
-          s_expert_of[s] = e;
-          s_slot_of[e] = s;
-          d.miss_list[(u / S) * S + wave_miss] = u;
-        }
-        ++wave_miss;
-        ++misses;
-      } else {
-        ++hits;
-      }
-      if (lane == 0 && (u % S == S - 1 || u == U - 1)) d.info[2 + u / S] = wave_miss;
-      if (lane == 0) {
-        s_last[s] = ++clock;
-        s_uslot[u] = s;
-        d.uniq[u] = e;
-        d.uslot[u] = s;
-        d.umiss[u] = hit ? 0 : 1;
-        d.tr_expert[(size_t)layer * E + u] = e;
-        d.tr_slot[(size_t)layer * E + u] = s;
-        d.tr_hit[(size_t)layer * E + u] = hit ? 1 : 0;
-      }
-      __syncwarp();  // lane 0's shared-memory updates are seen by the whole warp next access
-    }
-    if (lane == 0) {
-      d.clock[layer] = clock;
-      uint64_t* st = d.stats + (size_t)layer * 5;
-      st[0] += (uint64_t)U;
-      st[1] += hits;
-      st[2] += misses;
-      st[3] += evictions;
-      st[4] += misses * d.lay.canonical;
-      d.info[0] = U;
-      d.info[1] = (U + S - 1) / S;
-      d.tr_n[layer] = U;
-    }
-  }
+  if (warp == 0) lru_warp(d, layer, U, s_uniq, s_slot_of, s_expert_of, s_last, s_uslot);
   __syncthreads();
   for (int p = tid; p < n; p += nt) d.pos_slot[p] = s_uslot[uidx[d.idx[p]]];
   for (int e = tid; e < E; e += nt) g_slot_of[e] = s_slot_of[e];

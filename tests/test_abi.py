@@ -8,14 +8,14 @@ import pytest
 
 import oracle
 import synth
-from paper_2607_09686_gb300 import _build
+import __graft_entry__
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
 @pytest.fixture(scope="module")
 def mf():
-    _build.build()
+    __graft_entry__.build()
     import paper_2607_09686_gb300 as pkg
     return pkg
 

@@ -50,6 +50,7 @@ def _decode_run(shape, slots, n_tokens, seed, route=None, layers=None, sample_y=
                                             ctx.wr_host[l], b, xs[l][t:t + 1])
                     assert_outputs_close(y, yo, f"layer {l} token {t}")
                     n_checked += 1
+        assert ctx.mf.mf_check(ctx.h) == 0
         for l in layers:
             st = ctx.mf.mf_stats(ctx.h, l)
             ost = lru[l].stats()
@@ -72,11 +73,22 @@ def test_l4e64_decode(pct):
     _decode_run(Shape.of(cfg), S, cfg.n_tokens, seed=0, route=cfg.route_classes[0], sample_y=48)
 
 
+@pytest.mark.parametrize("kernels", ["pipelined", "simple"])
 @pytest.mark.parametrize("qtype", [synth.Q8_0, synth.Q4_0])
-def test_ragged_shapes_decode(qtype):
-    """Rows of 6 / 10 (Q8_0) and 3 / 5 (Q4_0) 16-byte vectors: partially filled warps."""
+def test_ragged_shapes_decode(qtype, kernels, monkeypatch):
+    """Rows of 6 / 10 (Q8_0) and 3 / 5 (Q4_0) 16-byte vectors: partially filled warps.  Both the
+    pipelined batch-1 kernels and the one-warp-per-row kernels (used for shapes the pipelined ones
+    do not take) are checked."""
+    if kernels == "simple":
+        monkeypatch.setenv("MF_DECODE_SIMPLE", "1")
     shape = Shape(2, 96, 12, 3, 160, qtype, model_seed=5)
     _decode_run(shape, 4, 40, seed=3)
+
+
+def test_q4_0_decode_full_width():
+    """Q4_0 at hidden 2048 / intermediate 768 (the 48-layer Q4_0 shape), one layer, batch 1."""
+    shape = Shape(1, 2048, 128, 8, 768, synth.Q4_0, model_seed=0)
+    _decode_run(shape, 19, 24, seed=2, route=synth.configs.ZIPF12, sample_y=12)
 
 
 def _batch_run(shape, slots, T, n_steps, seed, zipf_s=1.0, layers=None, sample_tokens=None):
