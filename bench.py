@@ -142,12 +142,12 @@ def run_mawforge(args):
 
     # one graph per step (the 1024 calls of a 256-token sequence), captured through the C ABI with
     # the library's per-kernel event records inside, so the kernel times come from the timed replays
-    mf.mf_timing(ctx, True)
+    timed = ["materialize", "gateup_swiglu", "down_combine"]
     graph = torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
         step_calls()  # untimed eager pass: warms the pool
         stream.synchronize()
-        mf.mf_timing(ctx, True)
+        mf.mf_timing(ctx, timed)
         with torch.cuda.graph(graph, stream=stream):
             step_calls()
     torch.cuda.synchronize()
@@ -185,7 +185,7 @@ def run_mawforge(args):
         torch.distributed.barrier()
         ms = float(t.item())
     st = mf.mf_stats(ctx, -1)  # every step starts cold (mf_reset), so these are one step's counters
-    mf.mf_timing(ctx, False)
+    mf.mf_timing(ctx, [])
 
     # end to end through the host-buffer entry point: per token, pinned host x/bias in, y out
     xh = torch.from_numpy(x_np).pin_memory()

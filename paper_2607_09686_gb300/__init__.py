@@ -73,7 +73,7 @@ _sig = {
     "mf_stats": (_i32, [_vp, _i32, ctypes.POINTER(Stats), _i32]),
     "mf_reset": (_i32, [_vp, _i32, _vp]),
     "mf_trace": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, ctypes.POINTER(_i32)]),
-    "mf_timing": (_i32, [_vp, _i32]),
+    "mf_timing": (_i32, [_vp, ctypes.c_uint]),
     "mf_timing_read": (_i32, [_vp, _vp, _vp]),
     "mf_check": (_i32, [_vp]),
     "mf_destroy": (None, [_vp]),
@@ -196,8 +196,17 @@ def mf_trace(ctx: int, layer: int, cap: int = 1024):
     return list(exp[:n.value]), list(slo[:n.value]), [bool(v) for v in hit[:n.value]]
 
 
-def mf_timing(ctx: int, enable: bool) -> None:
-    _check(_lib.mf_timing(ctx, 1 if enable else 0), "mf_timing")
+def mf_timing(ctx: int, classes=None) -> None:
+    """Time the kernel classes named in `classes` (names from KERNEL_CLASSES; None = all, [] = off)."""
+    if classes is None:
+        mask = (1 << len(KERNEL_CLASSES)) - 1
+    elif classes is False:
+        mask = 0
+    else:
+        mask = 0
+        for c in classes:
+            mask |= 1 << KERNEL_CLASSES.index(c)
+    _check(_lib.mf_timing(ctx, mask), "mf_timing")
 
 
 def mf_timing_read(ctx: int) -> dict:

@@ -137,7 +137,7 @@ uint64_t overhead_bytes(const mf_model_t& m, int S, int Tm) {
 
 // ---- per-kernel event timing
 void timer_mark(mf_ctx* c, int cls, int which, cudaStream_t s) {
-  if (!c->timing) return;
+  if (!(c->timing & (1u << cls))) return;
   int n = c->timer_n[cls];
   if (n >= c->timer_cap) {
     if (which == 1) c->timer_dropped++;
@@ -182,7 +182,8 @@ void free_ctx(mf_ctx* c) {
   delete c;
 }
 
-// repack one canonical GGUF tensor [rows x cols] into codes + scales
+// repack one canonical GGUF tensor [rows x cols] into codes + scales; Q8_0 codes are stored
+// offset to unsigned (q + 128), which the dequantising kernels expect
 void repack_tensor(const uint8_t* src, int rows, int cols, int qtype, uint8_t* codes, uint8_t* scales) {
   const int nb = cols / 32;
   const int bb = (int)block_bytes(qtype);
@@ -193,7 +194,11 @@ void repack_tensor(const uint8_t* src, int rows, int cols, int qtype, uint8_t* c
       uint8_t* sc = scales + ((size_t)r * nb + b) * 2;
       sc[0] = blk[0];
       sc[1] = blk[1];
-      memcpy(codes + ((size_t)r * nb + b) * cb, blk + 2, (size_t)cb);
+      uint8_t* dst = codes + ((size_t)r * nb + b) * cb;
+      if (qtype == MF_Q8_0)
+        for (int i = 0; i < cb; ++i) dst[i] = (uint8_t)(blk[2 + i] ^ 0x80u);  // q + 128, unsigned
+      else
+        memcpy(dst, blk + 2, (size_t)cb);
     }
   }
 }
@@ -583,8 +588,9 @@ int mf_trace(mf_ctx_t* c, int layer, int32_t* experts, int32_t* slots, uint8_t* 
   return MF_OK;
 }
 
-int mf_timing(mf_ctx_t* c, int enable) {
+int mf_timing(mf_ctx_t* c, unsigned class_mask) {
   if (!c) return MF_E_INVAL;
+  const unsigned enable = class_mask & ((1u << kTimerClasses) - 1);
   DevGuard guard(c->device);
   if (!guard.ok) return cuda_fail(cudaSetDevice(c->device), "cudaSetDevice");
   if (enable && !c->timer_ev[0]) {
@@ -598,7 +604,7 @@ int mf_timing(mf_ctx_t* c, int enable) {
   MF_CUDA(cudaDeviceSynchronize());
   for (int i = 0; i < kTimerClasses; ++i) c->timer_n[i] = 0;
   c->timer_dropped = 0;
-  c->timing = enable ? 1 : 0;
+  c->timing = enable;
   return MF_OK;
 }
 

@@ -15,8 +15,8 @@ constexpr int kTimerClasses = 6;
 enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5 };
 
 // SoA layout of one expert slot, identical in the pinned pack and in the HBM pool.
-// Quantised codes of each tensor are contiguous row-major (Q8_0: 1 byte per weight,
-// Q4_0: the 16 code bytes of each block in GGUF order), scales are binary16 row-major
+// Quantised codes of each tensor are contiguous row-major (Q8_0: 1 byte per weight, stored as
+// q + 128; Q4_0: the 16 code bytes of each block in GGUF order), scales are binary16 row-major
 // [rows][cols/32].  Every region starts on a 256-byte boundary.
 struct Layout {
   uint64_t gq, uq, dq;  // byte offsets of the gate / up / down codes
@@ -137,7 +137,7 @@ struct mf_ctx {
   int32_t* stage_idx;
   float* stage_w;
   // event timing
-  int timing;
+  unsigned timing;  // bit i set: kernel class i is timed
   int timer_cap;
   int timer_n[mf::kTimerClasses];
   int64_t timer_dropped;

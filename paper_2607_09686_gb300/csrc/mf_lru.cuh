@@ -17,9 +17,8 @@ namespace mf {
 // Writes the call's access record (uniq, uslot, umiss, trace), per-wave miss lists and counts,
 // the counters and the clock.  All 32 lanes must call it; lane 0 does the writes.
 __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const int* s_uniq, int* s_slot_of,
-                                         int* s_expert_of, uint64_t* s_last, int* s_uslot) {
-  const int lane = threadIdx.x & 31, E = d.E, S = d.S_active;
-  uint64_t clock = d.clock[layer];  // kept by lane 0
+                                         int* s_expert_of, uint64_t* s_last, int* s_uslot, uint64_t clock) {
+  const int lane = threadIdx.x & 31, E = d.E, S = d.S_active;  // the clock is kept by lane 0
   uint64_t hits = 0, misses = 0, evictions = 0;
   int wave_miss = 0;
   for (int u = 0; u < U; ++u) {
@@ -81,12 +80,12 @@ __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const i
   }
   if (lane == 0) {
     d.clock[layer] = clock;
-    uint64_t* st = d.stats + (size_t)layer * 5;
-    st[0] += (uint64_t)U;
-    st[1] += hits;
-    st[2] += misses;
-    st[3] += evictions;
-    st[4] += misses * d.lay.canonical;
+    unsigned long long* st = reinterpret_cast<unsigned long long*>(d.stats + (size_t)layer * 5);
+    atomicAdd(st + 0, (unsigned long long)U);  // no return value used: fire-and-forget reductions
+    atomicAdd(st + 1, (unsigned long long)hits);
+    atomicAdd(st + 2, (unsigned long long)misses);
+    atomicAdd(st + 3, (unsigned long long)evictions);
+    atomicAdd(st + 4, (unsigned long long)(misses * d.lay.canonical));
     d.info[0] = U;
     d.info[1] = (U + S - 1) / S;
     d.tr_n[layer] = U;

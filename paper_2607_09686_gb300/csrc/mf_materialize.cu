@@ -4,8 +4,8 @@
 // The misses are decided on the device (slot resolve), so the copy is driven by the GPU
 // itself: SMs load 16-byte vectors straight from the pinned, device-mapped pack over the
 // CPU-GPU link and store them into the slot, with no host round trip.  Launched on the
-// context's side stream.  Grid (chunks, max misses of the wave); block m copies part of
-// miss m of the wave, blocks past the wave's miss count exit at once.
+// context's side stream, two blocks per SM striding over the (miss, vector) pairs of the
+// wave; with no miss every block returns at once.
 #include "mf_internal.cuh"
 
 namespace mf {
@@ -14,25 +14,30 @@ namespace {
 constexpr int kUnroll = 8;
 
 __global__ void __launch_bounds__(256) k_materialize(Dev d, int layer, int wave) {
-  const int m = blockIdx.y;
-  if (m >= d.info[2 + wave]) return;
-  const int u = d.miss_list[wave * d.S_active + m];
-  const int e = d.uniq[u], s = d.uslot[u];
-  const uint4* src = reinterpret_cast<const uint4*>(d.pack + ((size_t)layer * d.E + e) * d.lay.stride);
-  uint4* dst = reinterpret_cast<uint4*>(d.pool + ((size_t)layer * d.S_alloc + s) * d.lay.stride);
-  const size_t nvec = d.lay.stride / 16;
+  const int n_miss = d.info[2 + wave];
+  if (n_miss == 0) return;
+  const size_t nvec = d.lay.stride / 16;  // 16-byte vectors per payload
+  const size_t total = (size_t)n_miss * nvec;
   const size_t step = (size_t)gridDim.x * blockDim.x * kUnroll;
-  for (size_t i = (size_t)blockIdx.x * blockDim.x * kUnroll + threadIdx.x; i < nvec; i += step) {
+  for (size_t i0 = (size_t)blockIdx.x * blockDim.x * kUnroll + threadIdx.x; i0 < total; i0 += step) {
     uint4 v[kUnroll];
 #pragma unroll
-    for (int r = 0; r < kUnroll; ++r) {
-      size_t j = i + (size_t)r * blockDim.x;
-      if (j < nvec) v[r] = ld_stream(src + j);
+    for (int r = 0; r < kUnroll; ++r) {  // all loads first: up to kUnroll transfers in flight per thread
+      const size_t i = i0 + (size_t)r * blockDim.x;
+      if (i < total) {
+        const int u = d.miss_list[wave * d.S_active + (int)(i / nvec)];
+        const uint8_t* src = d.pack + ((size_t)layer * d.E + d.uniq[u]) * d.lay.stride;
+        v[r] = ld_stream(src + 16 * (i % nvec));
+      }
     }
 #pragma unroll
     for (int r = 0; r < kUnroll; ++r) {
-      size_t j = i + (size_t)r * blockDim.x;
-      if (j < nvec) dst[j] = v[r];
+      const size_t i = i0 + (size_t)r * blockDim.x;
+      if (i < total) {
+        const int u = d.miss_list[wave * d.S_active + (int)(i / nvec)];
+        uint8_t* dst = d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride;
+        *reinterpret_cast<uint4*>(dst + 16 * (i % nvec)) = v[r];
+      }
     }
   }
 }
@@ -41,15 +46,15 @@ __global__ void __launch_bounds__(256) k_materialize(Dev d, int layer, int wave)
 
 cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s) {
   if (max_miss <= 0) return cudaSuccess;
-  const size_t nvec = d.lay.stride / 16;
-  const size_t per_block = (size_t)256 * kUnroll;
-  size_t chunks = (nvec + per_block - 1) / per_block;
-  // enough blocks in flight to cover the link latency even when one expert misses
-  size_t want = 4 * 152 / (size_t)max_miss;
-  if (want < 64) want = 64;
-  if (chunks > want) chunks = want;
-  dim3 grid((unsigned)chunks, (unsigned)max_miss);
-  k_materialize<<<grid, 256, 0, s>>>(d, layer, wave);
+  static int n_sm = 0;
+  if (!n_sm) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (n_sm <= 0) n_sm = 1;
+  }
+  // two blocks per SM stream all misses of the wave; the CPU-GPU link saturates well below this
+  k_materialize<<<2 * n_sm, 256, 0, s>>>(d, layer, wave);
   return cudaGetLastError();
 }
 

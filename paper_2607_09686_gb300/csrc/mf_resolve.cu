@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(256) k_resolve(Dev d, int layer, int T) {
   }
 
   // LRU, one access at a time
-  if (warp == 0) lru_warp(d, layer, U, s_uniq, s_slot_of, s_expert_of, s_last, s_uslot);
+  if (warp == 0) lru_warp(d, layer, U, s_uniq, s_slot_of, s_expert_of, s_last, s_uslot, d.clock[layer]);
   __syncthreads();
   for (int p = tid; p < n; p += nt) d.pos_slot[p] = s_uslot[uidx[d.idx[p]]];
   for (int e = tid; e < E; e += nt) g_slot_of[e] = s_slot_of[e];
