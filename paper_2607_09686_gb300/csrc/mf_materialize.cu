@@ -4,8 +4,8 @@
 // The misses are decided on the device (slot resolve), so the copy is driven by the GPU
 // itself: SMs load 16-byte vectors straight from the pinned, device-mapped pack over the
 // CPU-GPU link and store them into the slot, with no host round trip.  Launched on the
-// context's side stream, two blocks per SM striding over the (miss, vector) pairs of the
-// wave; with no miss every block returns at once.
+// context's side stream: two blocks per SM stride over each missed payload of the wave in
+// turn; with no miss every block returns at once.
 #include "mf_internal.cuh"
 
 namespace mf {
@@ -15,28 +15,23 @@ constexpr int kUnroll = 8;
 
 __global__ void __launch_bounds__(256) k_materialize(Dev d, int layer, int wave) {
   const int n_miss = d.info[2 + wave];
-  if (n_miss == 0) return;
   const size_t nvec = d.lay.stride / 16;  // 16-byte vectors per payload
-  const size_t total = (size_t)n_miss * nvec;
   const size_t step = (size_t)gridDim.x * blockDim.x * kUnroll;
-  for (size_t i0 = (size_t)blockIdx.x * blockDim.x * kUnroll + threadIdx.x; i0 < total; i0 += step) {
-    uint4 v[kUnroll];
+  for (int m = 0; m < n_miss; ++m) {
+    const int u = d.miss_list[wave * d.S_active + m];
+    const uint4* src = reinterpret_cast<const uint4*>(d.pack + ((size_t)layer * d.E + d.uniq[u]) * d.lay.stride);
+    uint4* dst = reinterpret_cast<uint4*>(d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride);
+    for (size_t i0 = (size_t)blockIdx.x * blockDim.x * kUnroll + threadIdx.x; i0 < nvec; i0 += step) {
+      uint4 v[kUnroll];
 #pragma unroll
-    for (int r = 0; r < kUnroll; ++r) {  // all loads first: up to kUnroll transfers in flight per thread
-      const size_t i = i0 + (size_t)r * blockDim.x;
-      if (i < total) {
-        const int u = d.miss_list[wave * d.S_active + (int)(i / nvec)];
-        const uint8_t* src = d.pack + ((size_t)layer * d.E + d.uniq[u]) * d.lay.stride;
-        v[r] = ld_stream(src + 16 * (i % nvec));
+      for (int r = 0; r < kUnroll; ++r) {  // all loads first: kUnroll transfers in flight per thread
+        const size_t i = i0 + (size_t)r * blockDim.x;
+        if (i < nvec) v[r] = ld_stream(src + i);
       }
-    }
 #pragma unroll
-    for (int r = 0; r < kUnroll; ++r) {
-      const size_t i = i0 + (size_t)r * blockDim.x;
-      if (i < total) {
-        const int u = d.miss_list[wave * d.S_active + (int)(i / nvec)];
-        uint8_t* dst = d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride;
-        *reinterpret_cast<uint4*>(dst + 16 * (i % nvec)) = v[r];
+      for (int r = 0; r < kUnroll; ++r) {
+        const size_t i = i0 + (size_t)r * blockDim.x;
+        if (i < nvec) dst[i] = v[r];
       }
     }
   }
