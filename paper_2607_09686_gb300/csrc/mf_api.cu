@@ -182,19 +182,21 @@ void free_ctx(mf_ctx* c) {
   delete c;
 }
 
-// repack one canonical GGUF tensor [rows x cols] into codes + scales; Q8_0 codes are stored
-// offset to unsigned (q + 128), which the dequantising kernels expect
-void repack_tensor(const uint8_t* src, int rows, int cols, int qtype, uint8_t* codes, uint8_t* scales) {
+// Repack one canonical GGUF tensor [rows x cols] into row records: the codes of row r go to
+// rec0 + r * rstride + codes_off, its binary16 scales to rec0 + r * rstride + scales_off.
+// Q8_0 codes are stored offset to unsigned (q + 128), which the dequantising kernels expect.
+void repack_tensor(const uint8_t* src, int rows, int cols, int qtype, uint8_t* rec0, uint32_t rstride,
+                   uint32_t codes_off, uint32_t scales_off) {
   const int nb = cols / 32;
   const int bb = (int)block_bytes(qtype);
   const int cb = qtype == MF_Q8_0 ? 32 : 16;
   for (int r = 0; r < rows; ++r) {
+    uint8_t* rec = rec0 + (size_t)r * rstride;
     for (int b = 0; b < nb; ++b) {
       const uint8_t* blk = src + ((size_t)r * nb + b) * bb;
-      uint8_t* sc = scales + ((size_t)r * nb + b) * 2;
-      sc[0] = blk[0];
-      sc[1] = blk[1];
-      uint8_t* dst = codes + ((size_t)r * nb + b) * cb;
+      rec[scales_off + 2 * b] = blk[0];
+      rec[scales_off + 2 * b + 1] = blk[1];
+      uint8_t* dst = rec + codes_off + (size_t)b * cb;
       if (qtype == MF_Q8_0)
         for (int i = 0; i < cb; ++i) dst[i] = (uint8_t)(blk[2 + i] ^ 0x80u);  // q + 128, unsigned
       else
@@ -217,20 +219,14 @@ Layout make_layout(const mf_model_t& m) {
   l.qrow_d = m.qtype == MF_Q8_0 ? (int)I : (int)(I / 2);
   l.nb_gu = (int)(H / 32);
   l.nb_d = (int)(I / 32);
-  uint64_t off = 0;
-  l.gq = off;
-  off = align256(off + I * l.qrow_gu);
-  l.uq = off;
-  off = align256(off + I * l.qrow_gu);
-  l.dq = off;
-  off = align256(off + H * l.qrow_d);
-  l.gd = off;
-  off = align256(off + I * l.nb_gu * 2);
-  l.ud = off;
-  off = align256(off + I * l.nb_gu * 2);
-  l.dd = off;
-  off = align256(off + H * l.nb_d * 2);
-  l.stride = off;
+  l.o_up = (uint32_t)l.qrow_gu;
+  l.o_gs = 2u * l.qrow_gu;
+  l.o_us = l.o_gs + 2u * l.nb_gu;
+  l.rs_gu = (uint32_t)((l.o_us + 2u * l.nb_gu + 15) & ~15u);
+  l.o_ds = (uint32_t)l.qrow_d;
+  l.rs_d = (uint32_t)((l.qrow_d + 2u * l.nb_d + 15) & ~15u);
+  l.d_off = align256(I * l.rs_gu);
+  l.stride = align256(l.d_off + H * l.rs_d);
   l.canonical = canonical_payload_bytes(m);
   return l;
 }
@@ -420,12 +416,12 @@ int mf_pack_put(mf_ctx_t* c, int layer, int expert, const void* payload, uint64_
   if (bytes != l.canonical) return MF_E_INVAL;
   const mf_model_t& m = c->model;
   uint8_t* dst = c->pack_host + ((uint64_t)layer * c->d.E + expert) * l.stride;
-  memset(dst, 0, l.stride);  // padding between regions stays zero
+  memset(dst, 0, l.stride);  // padding stays zero
   const uint8_t* src = static_cast<const uint8_t*>(payload);
   const uint64_t tb_gu = (uint64_t)m.inter * (m.hidden / 32) * block_bytes(m.qtype);
-  repack_tensor(src, m.inter, m.hidden, m.qtype, dst + l.gq, dst + l.gd);
-  repack_tensor(src + tb_gu, m.inter, m.hidden, m.qtype, dst + l.uq, dst + l.ud);
-  repack_tensor(src + 2 * tb_gu, m.hidden, m.inter, m.qtype, dst + l.dq, dst + l.dd);
+  repack_tensor(src, m.inter, m.hidden, m.qtype, dst, l.rs_gu, 0, l.o_gs);
+  repack_tensor(src + tb_gu, m.inter, m.hidden, m.qtype, dst, l.rs_gu, l.o_up, l.o_us);
+  repack_tensor(src + 2 * tb_gu, m.hidden, m.inter, m.qtype, dst + l.d_off, l.rs_d, 0, l.o_ds);
   unsigned char* seen = &c->put_map[(size_t)layer * c->d.E + expert];
   if (__atomic_exchange_n(seen, (unsigned char)1, __ATOMIC_ACQ_REL) == 0) __atomic_fetch_add(&c->n_put, 1, __ATOMIC_ACQ_REL);
   return MF_OK;

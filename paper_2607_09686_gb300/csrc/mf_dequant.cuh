@@ -97,6 +97,105 @@ __device__ __forceinline__ float dot_vec(uint4 w, const XV<QT>& x) {
   return f2_sum(f2_add(a, b));
 }
 
+// ---- exact integer dot products for vectors held in registers across many rows
+//
+// A vector of kW fp32 values v (x, or h) is split once into three int8 pieces
+//   v ~= s * (p1 + p2 / 127 + p3 / 127^2),  s = max|v| / 127,
+// so that |v - that| <= max|v| * 2^-22.  A row's codes c then give the exact integer sums
+// P_i = sum_j c_j p_i[j] with dp4a (4 byte products per instruction), and
+//   sum_j (c_j - off) v_j ~= s * ((P1 * 127 + P2 - off * (S1 * 127 + S2)) * 127 + P3 - off * S3) / 127^2
+// where S_i = sum_j p_i[j] and off is the code offset (128 for Q8_0's stored q + 128, 8 for Q4_0).
+// Every integer sum is exact (|P1 * 127| < 2^27); fp32 rounds only the final combination.
+template <int QT>
+struct XQ {
+  static constexpr int kWords = Vec<QT>::kW / 4;  // words of four values: 4 (Q8_0) or 8 (Q4_0)
+  uint32_t p1[kWords], p2[kWords], p3[kWords];
+  int k12, k3;  // offset corrections: off * (S1 * 127 + S2), off * S3
+  float sf;     // s / 127^2
+};
+
+template <int QT>
+__device__ __forceinline__ XQ<QT> quant_vec(const float* __restrict__ vp) {
+  constexpr int kW = Vec<QT>::kW;
+  float v[kW];
+#pragma unroll
+  for (int i = 0; i < kW / 4; ++i) {
+    const float4 f = __ldg(reinterpret_cast<const float4*>(vp) + i);
+    v[4 * i] = f.x;
+    v[4 * i + 1] = f.y;
+    v[4 * i + 2] = f.z;
+    v[4 * i + 3] = f.w;
+  }
+  float m = 0.f;
+#pragma unroll
+  for (int j = 0; j < kW; ++j) m = fmaxf(m, fabsf(v[j]));
+  const float inv = m > 0.f ? 127.f / m : 0.f;
+  XQ<QT> r;
+  int s1 = 0, s2 = 0, s3 = 0;
+#pragma unroll
+  for (int w = 0; w < XQ<QT>::kWords; ++w) {
+    uint32_t b1 = 0, b2 = 0, b3 = 0;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float t = v[4 * w + j] * inv;
+      const int a = __float2int_rn(t);
+      const float e = (t - (float)a) * 127.f;
+      const int b = __float2int_rn(e);
+      const int c = __float2int_rn((e - (float)b) * 127.f);
+      s1 += a;
+      s2 += b;
+      s3 += c;
+      b1 |= (uint32_t)(a & 0xFF) << (8 * j);
+      b2 |= (uint32_t)(b & 0xFF) << (8 * j);
+      b3 |= (uint32_t)(c & 0xFF) << (8 * j);
+    }
+    r.p1[w] = b1;
+    r.p2[w] = b2;
+    r.p3[w] = b3;
+  }
+  constexpr int off = QT == kQ8 ? 128 : 8;
+  r.k12 = off * (s1 * 127 + s2);
+  r.k3 = off * s3;
+  r.sf = m / 127.f / 16129.f;
+  return r;
+}
+
+// sum of four unsigned byte x signed byte products, added to c
+__device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
+  int d;
+  asm("dp4a.u32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
+// unscaled dot product of one code vector with a split vector
+template <int QT>
+__device__ __forceinline__ float dot_q(uint4 w, const XQ<QT>& x) {
+  int a = 0, b = 0, c = 0;
+  const uint32_t ws[4] = {w.x, w.y, w.z, w.w};
+  if constexpr (QT == kQ8) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      a = dp4a_us(ws[i], x.p1[i], a);
+      b = dp4a_us(ws[i], x.p2[i], b);
+      c = dp4a_us(ws[i], x.p3[i], c);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {  // byte j: element j (low nibble), element j + 16 (high nibble)
+      const uint32_t lo = ws[i] & 0x0F0F0F0Fu, hi = (ws[i] >> 4) & 0x0F0F0F0Fu;
+      a = dp4a_us(lo, x.p1[i], a);
+      a = dp4a_us(hi, x.p1[4 + i], a);
+      b = dp4a_us(lo, x.p2[i], b);
+      b = dp4a_us(hi, x.p2[4 + i], b);
+      c = dp4a_us(lo, x.p3[i], c);
+      c = dp4a_us(hi, x.p3[4 + i], c);
+    }
+  }
+  const int p12 = a * 127 + b - x.k12;
+  const int p3 = c - x.k3;
+  return fmaf((float)p12, 127.f, (float)p3) * x.sf;
+}
+
 template <int QT>
 __device__ __forceinline__ int scale_index(int v) {
   return QT == kQ8 ? (v >> 1) : v;

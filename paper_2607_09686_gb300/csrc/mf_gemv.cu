@@ -35,10 +35,10 @@ __global__ void __launch_bounds__(256) k_gateup(Dev d, int layer, int wave, cons
   const int r = blockIdx.x * 8 + warp;
   if (r >= d.I) return;
   const uint8_t* slot = slot_base(d, layer, d.uslot[u]);
-  const uint8_t* gq = slot + d.lay.gq + (size_t)r * d.lay.qrow_gu;
-  const uint8_t* uq = slot + d.lay.uq + (size_t)r * d.lay.qrow_gu;
-  const __half* gd = reinterpret_cast<const __half*>(slot + d.lay.gd) + (size_t)r * d.lay.nb_gu;
-  const __half* ud = reinterpret_cast<const __half*>(slot + d.lay.ud) + (size_t)r * d.lay.nb_gu;
+  const uint8_t* gq = slot + (size_t)r * d.lay.rs_gu;  // row record: gate, up codes; gate, up scales
+  const uint8_t* uq = gq + d.lay.o_up;
+  const __half* gd = reinterpret_cast<const __half*>(gq + d.lay.o_gs);
+  const __half* ud = reinterpret_cast<const __half*>(gq + d.lay.o_us);
   const int nvec = d.lay.qrow_gu / 16;
 
   uint4 wg[VPL], wu[VPL];
@@ -90,8 +90,8 @@ __global__ void __launch_bounds__(256) k_down_single(Dev d, int layer, float* __
       const int j = j0 + jj;
       if (j < k) {
         const uint8_t* slot = slot_base(d, layer, d.pos_slot[j]);
-        const uint8_t* q = slot + d.lay.dq + (size_t)c * d.lay.qrow_d;
-        const __half* s = reinterpret_cast<const __half*>(slot + d.lay.dd) + (size_t)c * d.lay.nb_d;
+        const uint8_t* q = slot + d.lay.d_off + (size_t)c * d.lay.rs_d;
+        const __half* s = reinterpret_cast<const __half*>(q + d.lay.o_ds);
 #pragma unroll
         for (int i = 0; i < VPL; ++i) {
           const int v = lane + 32 * i;
@@ -131,8 +131,8 @@ __global__ void __launch_bounds__(256) k_down_partial(Dev d, int layer, int wave
   const int c = blockIdx.x * 8 + warp;
   if (c >= d.H) return;
   const uint8_t* slot = slot_base(d, layer, d.uslot[u]);
-  const uint8_t* q = slot + d.lay.dq + (size_t)c * d.lay.qrow_d;
-  const __half* s = reinterpret_cast<const __half*>(slot + d.lay.dd) + (size_t)c * d.lay.nb_d;
+  const uint8_t* q = slot + d.lay.d_off + (size_t)c * d.lay.rs_d;
+  const __half* s = reinterpret_cast<const __half*>(q + d.lay.o_ds);
   const int nvec = d.lay.qrow_d / 16;
   uint4 w[VPL];
   float sc[VPL];

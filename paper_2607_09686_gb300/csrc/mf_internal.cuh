@@ -14,13 +14,17 @@ constexpr int kMaxExperts = 1024;
 constexpr int kTimerClasses = 6;
 enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5 };
 
-// SoA layout of one expert slot, identical in the pinned pack and in the HBM pool.
-// Quantised codes of each tensor are contiguous row-major (Q8_0: 1 byte per weight, stored as
-// q + 128; Q4_0: the 16 code bytes of each block in GGUF order), scales are binary16 row-major
-// [rows][cols/32].  Every region starts on a 256-byte boundary.
+// Layout of one expert slot, identical in the pinned pack and in the HBM pool: row records.
+// Gate/up region: I records, record r = [gate codes row r | up codes row r | gate scales row r
+// | up scales row r], padded to 16 bytes.  Down region: H records, record c = [down codes row c
+// | down scales row c], padded to 16 bytes.  Codes: Q8_0 one byte per weight stored as
+// q + 128; Q4_0 the 16 code bytes of each block in GGUF order.  Scales: binary16, one per 32
+// weights.  Rows that are computed together are contiguous, so a work item is one copy.
 struct Layout {
-  uint64_t gq, uq, dq;  // byte offsets of the gate / up / down codes
-  uint64_t gd, ud, dd;  // byte offsets of the gate / up / down scales
+  uint64_t d_off;       // byte offset of the down region (the gate/up region starts at 0)
+  uint32_t rs_gu, rs_d;  // bytes per gate/up record and per down record
+  uint32_t o_up, o_gs, o_us;  // inside a gate/up record: up codes, gate scales, up scales
+  uint32_t o_ds;        // inside a down record: scales
   uint64_t stride;      // bytes per slot (a multiple of 256)
   uint64_t canonical;   // canonical GGUF payload bytes (what a miss accounts for)
   int qrow_gu, qrow_d;  // code bytes per row: gate/up rows (hidden weights), down rows (inter weights)
