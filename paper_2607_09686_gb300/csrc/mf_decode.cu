@@ -44,13 +44,16 @@ struct PipeCfg {
   int cs;                // gate/up: column ranges per row (16 / (2R))
   int max_mine;          // most items any block gets
   int slots;             // partial results per item
+  int n_vec;             // vectors split into int8 pieces at kernel start (x, or the k h's)
+  uint32_t vq_bytes;     // their shared-memory bytes
 };
 
 struct Smem {
   unsigned char* stage0;
   uint64_t* full;
   uint64_t* empty;
-  float* red;  // [max_mine][16 warps]: every partial result of the block, combined at the end
+  float* red;         // [max_mine][16 warps]: every partial result of the block, combined at the end
+  unsigned char* vq;  // [n_vec] split vectors (XQ), written once by the consumers at kernel start
 };
 
 __device__ __forceinline__ Smem carve(unsigned char* base, const PipeCfg& c) {
@@ -60,13 +63,22 @@ __device__ __forceinline__ Smem carve(unsigned char* base, const PipeCfg& c) {
   s.full = reinterpret_cast<uint64_t*>(p);
   s.empty = s.full + kMaxStages;
   s.red = reinterpret_cast<float*>(s.empty + kMaxStages);
+  s.vq = reinterpret_cast<unsigned char*>(s.red + c.max_mine * kConsumers);
   return s;
 }
 
 size_t part_bytes(int max_mine) { return (size_t)max_mine * kConsumers * sizeof(float); }
 
 size_t smem_bytes(const PipeCfg& c) {
-  return (size_t)c.NS * c.stage_bytes + 2 * kMaxStages * sizeof(uint64_t) + part_bytes(c.max_mine);
+  return (size_t)c.NS * c.stage_bytes + 2 * kMaxStages * sizeof(uint64_t) + part_bytes(c.max_mine) + c.vq_bytes;
+}
+
+// The consumers split `n` vectors of kW values into int8 pieces, one vector per thread, into
+// shared memory, then wait for each other (the producer keeps streaming meanwhile).
+template <int QT>
+__device__ __forceinline__ void split_vectors(const float* __restrict__ src, int n, XQ<QT>* dst) {
+  for (int i = threadIdx.x; i < n; i += kConsumers * 32) dst[i] = quant_vec<QT>(src + (size_t)i * Vec<QT>::kW);
+  named_bar_sync(1, kConsumers * 32);
 }
 
 // Items of this block: blockIdx.x, blockIdx.x + gridDim.x, ...  Producer and consumers both
@@ -150,11 +162,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, c
     const int ten = warp / (R * cs), row = (warp / cs) % R, col = warp % cs;
     const int nv = (qrow / 16) / cs;  // vectors in this warp's column range
     const int v0 = col * nv;
+    const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
+    split_vectors<QT>(x, c.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq));
     XQ<QT> xr[VPL];
 #pragma unroll
     for (int i = 0; i < VPL; ++i) {
       const int v = lane + 32 * i;
-      if (v < nv) xr[i] = quant_vec<QT>(x + (v0 + v) * Vec<QT>::kW);
+      if (v < nv) xr[i] = xq[v0 + v];
     }
     Ring ring;
     for (int it = 0; it < mine; ++it) {
@@ -240,12 +254,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
   } else {
     const int j = warp / R, rho = warp % R;  // one (expert, row) task per warp: k * R <= 16
     const bool active = j < k;
+    const XQ<QT>* hq = reinterpret_cast<const XQ<QT>*>(sm.vq);
+    split_vectors<QT>(d.h, c.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq));  // h of all k experts
     XQ<QT> hr[VPLD];
     if (active) {
 #pragma unroll
       for (int i = 0; i < VPLD; ++i) {
         const int v = lane + 32 * i;
-        if (v < nvec) hr[i] = quant_vec<QT>(d.h + (size_t)j * d.I + v * Vec<QT>::kW);
+        if (v < nvec) hr[i] = hq[j * nvec + v];
       }
     }
     Ring ring;
@@ -324,7 +340,9 @@ PipeCfg gateup_cfg(const Dev& d) {
   c.per_j = 0;
   c.slots = kConsumers;
   c.max_mine = (c.n_items + sm_count() - 1) / sm_count();
-  c.NS = stages_for(c.stage_bytes, part_bytes(c.max_mine));
+  c.n_vec = d.lay.qrow_gu / 16;
+  c.vq_bytes = (uint32_t)(c.n_vec * (d.qtype == MF_Q8_0 ? sizeof(XQ<kQ8>) : sizeof(XQ<kQ4>)));
+  c.NS = stages_for(c.stage_bytes, part_bytes(c.max_mine) + c.vq_bytes);
   return c;
 }
 
@@ -337,7 +355,9 @@ PipeCfg down_cfg(const Dev& d) {
   c.n_items = d.H / c.R;
   c.slots = kConsumers;
   c.max_mine = (c.n_items + sm_count() - 1) / sm_count();
-  c.NS = stages_for(c.stage_bytes, part_bytes(c.max_mine));
+  c.n_vec = d.k * (d.lay.qrow_d / 16);
+  c.vq_bytes = (uint32_t)(c.n_vec * (d.qtype == MF_Q8_0 ? sizeof(XQ<kQ8>) : sizeof(XQ<kQ4>)));
+  c.NS = stages_for(c.stage_bytes, part_bytes(c.max_mine) + c.vq_bytes);
   return c;
 }
 
