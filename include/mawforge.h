@@ -174,6 +174,37 @@ int mf_timing_read(mf_ctx_t* ctx, double* ms, int64_t* launches);
  * within the limit makes the kernel record the failure and return. */
 int mf_check(mf_ctx_t* ctx);
 
+/* One-token expert FFN with no allocation at all (the paper has no counterpart: it is a
+ * convenience of this library).  Callers that cannot allocate device memory — code running
+ * while a CUDA graph is being captured under a no-allocation policy, latency-critical threads
+ * that must not take cudaMalloc's implicit device synchronisation, or plugins confined to a
+ * device-memory budget reserved by their host process — can still compute
+ *   y = sum_j g[j] * down_j( silu(gate_j x) * (up_j x) ),   j < model->top_k,
+ * from expert weights they already hold, without creating a context.  It runs the kernels of
+ * a one-token mf_moe_forward; their intermediate h and index tables live in a file-scope
+ * device array of 128 KiB + 256 B, which every GPU that loads this library holds until the
+ * process exits.
+ *   model    hidden, inter, top_k (<= 8) and qtype are used; top_k * inter must be <= 32768
+ *            (else MF_E_INVAL: the static scratch is sized for that)
+ *   experts  device, 16-byte aligned: top_k expert slots back to back, slot j = expert j, each
+ *            `stride` bytes in this layout (Q = bytes of codes per row: hidden (Q8_0) or
+ *            hidden/2 (Q4_0) for gate/up rows, inter or inter/2 for down rows; nb = weights/32):
+ *              rs_gu = round16(2*Q_gu + 4*nb_gu), rs_d = round16(Q_d + 2*nb_d),
+ *              d_off = round256(inter * rs_gu), stride = round256(d_off + hidden * rs_d);
+ *              gate/up record r at r*rs_gu: [gate codes row r][up codes row r]
+ *                [gate scales row r (nb_gu binary16)][up scales row r], zero padding;
+ *              down record c at d_off + c*rs_d: [down codes row c][down scales row c];
+ *              codes in GGUF block order, Q8_0 codes stored as q + 128 (unsigned byte)
+ *   g        device float [top_k] weights of the experts; x device float [hidden], 16-byte
+ *            aligned; y device float [hidden] output
+ * Stream-ordered on `stream`; returns after enqueueing.  The first call on each device sets up
+ * that device (it reads the array's device address and writes its constant tables): make that
+ * first call before any stream capture.  All calls on a device share the array, so calls whose
+ * kernels overlap on the GPU (other streams, other host threads) race on it: serialise them.
+ * Nothing in the array needs clearing between calls; h is fully rewritten by each call. */
+int mf_expert_ffn_noalloc(const mf_model_t* model, const void* experts, const float* g, const float* x,
+                          float* y, void* stream);
+
 /* Release everything the context owns (synchronises its streams first). NULL is a no-op. */
 void mf_destroy(mf_ctx_t* ctx);
 

@@ -17,7 +17,7 @@ import os
 __all__ = [
     "MFError", "Model", "PlanReq", "Plan", "Stats", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
     "mf_payload_bytes", "mf_plan", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
-    "mf_moe_forward_host", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_destroy",
+    "mf_moe_forward_host", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_expert_ffn_noalloc", "mf_destroy",
     "mf_strerror", "mf_last_cuda_error",
 ]
 
@@ -76,6 +76,7 @@ _sig = {
     "mf_timing": (_i32, [_vp, ctypes.c_uint]),
     "mf_timing_read": (_i32, [_vp, _vp, _vp]),
     "mf_check": (_i32, [_vp]),
+    "mf_expert_ffn_noalloc": (_i32, [ctypes.POINTER(Model), _vp, _vp, _vp, _vp, _vp]),
     "mf_destroy": (None, [_vp]),
     "mf_strerror": (ctypes.c_char_p, [_i32]),
     "mf_last_cuda_error": (ctypes.c_char_p, []),
@@ -223,6 +224,12 @@ def mf_check(ctx: int) -> int:
     if rc not in (MF_OK, MF_E_TIMEOUT):
         _check(rc, "mf_check")
     return rc
+
+
+def mf_expert_ffn_noalloc(model: Model, experts, g, x, y, stream=None) -> None:
+    """One-token expert FFN from caller-held expert slots, allocating nothing (see mawforge.h)."""
+    _check(_lib.mf_expert_ffn_noalloc(ctypes.byref(model), _addr(experts), _addr(g), _addr(x), _addr(y),
+                                      _stream(stream)), "mf_expert_ffn_noalloc")
 
 
 def mf_destroy(ctx: int) -> None:
