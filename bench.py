@@ -32,6 +32,21 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "l4e64"
 N_TOKENS = 256
 
+# DRAM bytes (read + write) of one gate/up launch from the ncu capture summarised in
+# profiles/k_gateup_pipe_l4e64_decode.md, valid while the kernel sources hash to `sha`.
+GATEUP_TRAFFIC = {"sha": "81f6b54c28f8fe9f", "bytes": 26780672,
+                  "files": ("paper_2607_09686_gb300/csrc/mf_decode.cu", "paper_2607_09686_gb300/csrc/mf_dequant.cuh",
+                            "paper_2607_09686_gb300/csrc/mf_internal.cuh")}
+
+
+def _captured_traffic():
+    import hashlib
+    h = hashlib.sha256()
+    for f in GATEUP_TRAFFIC["files"]:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return GATEUP_TRAFFIC["bytes"] if h.hexdigest()[:16] == GATEUP_TRAFFIC["sha"] else None
+
 
 def _peaks():
     try:
@@ -258,7 +273,7 @@ def run_mawforge(args):
                   "misses_per_token": st["misses"] / N_TOKENS, "accesses_per_step": st["accesses"]},
         "roofline": {"bound": "hbm", "kernel": "gateup_swiglu (grouped dequant-GEMV, k experts' gate+up rows)",
                      "achieved": round(gu_gbs, 1), "peak": hbm, "unit": "GB/s",
-                     "frac": round(gu_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": None,
+                     "frac": round(gu_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": _captured_traffic(),
                      "gemv_pair_gbs": round(gemv_gbs, 1), "gemv_pair_frac": round(gemv_gbs / hbm, 4),
                      "frac_of_8tbs": round(gemv_gbs / 8000.0, 4),
                      "bytes_per_launch": {"gateup": gu_bytes, "down": dn_bytes}},
