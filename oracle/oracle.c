@@ -87,7 +87,7 @@ uint64_t orc_payload_bytes(int hidden, int inter, int qtype) {
 /* z_e = fp32(sum_i W[e,i] x_i) computed with exact fp64 products and fp64 summation,
  * then + bias_e in fp32.  Chosen: the k largest z, ties to the lower id, listed in that
  * order.  g_j = exp(z_j - z_max) / sum_chosen exp(z - z_max) in fp64. */
-static const float* g_sort_z;
+static _Thread_local const float* g_sort_z; /* per thread: the oracle may be called from several threads */
 static int cmp_desc(const void* a, const void* b) {
   int ia = *(const int*)a, ib = *(const int*)b;
   float za = g_sort_z[ia], zb = g_sort_z[ib];

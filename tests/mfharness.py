@@ -73,7 +73,7 @@ class Payloads:
 class Ctx:
     """A context of the CUDA library with its pack filled from the seeded generator."""
 
-    def __init__(self, shape: Shape, slots: int, max_tokens: int, device: int = 0, workers: int = 4):
+    def __init__(self, shape: Shape, slots: int, max_tokens: int, device: int = 0, workers: int = 8):
         import torch
         import paper_2607_09686_gb300 as mf
         self.mf, self.torch, self.s = mf, torch, shape
@@ -127,3 +127,37 @@ class Ctx:
 def oracle_trace(lru: oracle.LRU, idx: np.ndarray):
     u, sl, hit = lru.step(idx)
     return list(map(int, u)), list(map(int, sl)), list(map(bool, hit))
+
+
+def oracle_routes(shape: Shape, wr_host, xs, biases, workers: int = 16) -> np.ndarray:
+    """Oracle routing of many (layer, token) inputs, in a thread pool (the C oracle releases the
+    GIL).  xs[l] is [T, H], biases[l] is [T, E] or None; returns idx [L, T, k]."""
+    L = len(xs)
+    T = xs[0].shape[0]
+    out = np.empty((L, T, shape.top_k), np.int32)
+
+    def one(lt):
+        l, t = lt
+        b = None if biases[l] is None else biases[l][t]
+        out[l, t] = oracle.router(xs[l][t], wr_host[l], b, shape.top_k)[1]
+
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        list(ex.map(one, [(l, t) for l in range(L) for t in range(T)]))
+    return out
+
+
+def oracle_stats(shape: Shape, slots: int, idx_steps) -> list:
+    """Per-layer oracle LRU counters after feeding idx_steps[l] = list of [T_step, k] arrays."""
+    pay = synth.payload_bytes(shape.hidden, shape.inter, shape.qtype)
+    res = []
+    for steps in idx_steps:
+        c = oracle.LRU(shape.n_experts, slots, pay)
+        for st in steps:
+            c.step(st)
+        res.append(c.stats())
+    return res
+
+
+def stats_tuple(st: dict):
+    return (st["accesses"], st["hits"], st["misses"], st["evictions"],
+            st.get("bytes", st.get("bytes_materialized")))
