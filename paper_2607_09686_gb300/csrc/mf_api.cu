@@ -87,7 +87,7 @@ struct Carve {
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
   uint64_t logits, ticket, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
-  uint64_t work, err, sx, sb, sy, sidx, sw;
+  uint64_t work, err, xs, sx, sb, sy, sidx, sw;
   uint64_t total;
 };
 
@@ -120,6 +120,7 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.part = c.take<float>(Tm > 1 ? (uint64_t)Tm * k * H : 1);
   o.work = c.take<unsigned>(4);
   o.err = c.take<unsigned>(1);
+  o.xs = c.take<uint16_t>(Tm > 1 ? 2ull * Tm * H : 1);
   o.sx = c.take<float>((uint64_t)Tm * H);
   o.sb = c.take<float>((uint64_t)Tm * E);
   o.sy = c.take<float>((uint64_t)Tm * H);
@@ -367,6 +368,10 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.part = reinterpret_cast<float*>(base + so.part);
   d.work = reinterpret_cast<unsigned*>(base + so.work);
   d.err = reinterpret_cast<unsigned*>(base + so.err);
+  if (Tm > 1) {
+    d.xh = reinterpret_cast<uint16_t*>(base + so.xs);
+    d.xl = d.xh + (size_t)Tm * d.H;
+  }
   c->stage_x = reinterpret_cast<float*>(base + so.sx);
   c->stage_bias = reinterpret_cast<float*>(base + so.sb);
   c->stage_y = reinterpret_cast<float*>(base + so.sy);
@@ -406,6 +411,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
     return MF_E_INVAL;
   }
   c->decode_pipe = decode_pipe_ok(d) && getenv("MF_DECODE_SIMPLE") == nullptr;
+  c->prefill_min_t = Tm > 1 && prefill_shape_ok(d.H, d.I) ? kPrefillMinTokens : 0;
   *out = c;
   return MF_OK;
 }
@@ -468,6 +474,9 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
     timer_mark(c, kTResolve, 1, s);
   }
 
+  const bool gemm = T > 1 && c->prefill_min_t > 0 && T >= c->prefill_min_t;
+  if (gemm) MF_CUDA(launch_split_x(d, x, T, s));
+
   long long accesses_max = (long long)T * d.k;
   if (accesses_max > d.E) accesses_max = d.E;
   const int n_waves = (int)((accesses_max + S - 1) / S);
@@ -481,6 +490,18 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
     timer_mark(c, kTMaterialize, 1, c->side);
     MF_CUDA(cudaEventRecord(c->ev_join[w], c->side));
     MF_CUDA(cudaStreamWaitEvent(s, c->ev_join[w], 0));
+    if (gemm) {
+      timer_mark(c, kTPrefill, 0, s);
+      MF_CUDA(launch_prefill_gateup(d, layer, w, s));
+      MF_CUDA(launch_prefill_down(d, layer, w, s));
+      timer_mark(c, kTPrefill, 1, s);
+      if (w == n_waves - 1) {
+        timer_mark(c, kTDown, 0, s);
+        MF_CUDA(launch_combine(d, T, y, s));
+        timer_mark(c, kTDown, 1, s);
+      }
+      continue;
+    }
     const bool pipe = T == 1 && c->decode_pipe;
     timer_mark(c, kTGateUp, 0, s);
     if (pipe)
@@ -500,6 +521,13 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   }
   if (idx_out) MF_CUDA(cudaMemcpyAsync(idx_out, d.idx, sizeof(int32_t) * T * d.k, cudaMemcpyDeviceToDevice, s));
   if (w_out) MF_CUDA(cudaMemcpyAsync(w_out, d.g, sizeof(float) * T * d.k, cudaMemcpyDeviceToDevice, s));
+  return MF_OK;
+}
+
+int mf_prefill_threshold(mf_ctx_t* c, int min_tokens) {
+  if (!c || min_tokens < 0 || min_tokens == 1) return MF_E_INVAL;
+  if (min_tokens > 0 && (c->d.T_max < 2 || !prefill_shape_ok(c->d.H, c->d.I))) return MF_E_INVAL;
+  c->prefill_min_t = min_tokens;
   return MF_OK;
 }
 

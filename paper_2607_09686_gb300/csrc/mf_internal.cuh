@@ -66,6 +66,8 @@ struct Dev {
   int32_t* miss_list;  // [E + S_alloc] unique index of miss m of wave w at w * S_active + m
   float* h;            // [T_max * k][I]  SwiGLU activations
   float* part;         // [T_max * k][H]  per-assignment down outputs (T > 1)
+  uint16_t* xh;        // [T_max][H]    bf16 high part of x (tensor-core prefill path, T_max > 1)
+  uint16_t* xl;        // [T_max][H]    bf16 low part, x - hi
   unsigned* work;      // [4]           work-queue counters of the pipelined decode kernels
   unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
 };
@@ -148,6 +150,7 @@ struct mf_ctx {
   cudaEvent_t* timer_ev[mf::kTimerClasses];  // pairs: [2 * i], [2 * i + 1]
   uint64_t overhead_bytes;
   bool decode_pipe;  // batch-1 calls use the pipelined decode kernels
+  int prefill_min_t;  // calls with T >= this use the tensor-core grouped GEMMs (0 = never)
 };
 
 namespace mf {
@@ -171,5 +174,11 @@ cudaError_t launch_gateup_single(const Dev& d, int layer, const float* x, cudaSt
 cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStream_t s);
 size_t decode_smem_bytes(const Dev& d, int which);
 bool decode_pipe_ok(const Dev& d);
+// many tokens per expert: tcgen05 grouped GEMMs (gate/up + SwiGLU, down) per wave
+constexpr int kPrefillMinTokens = 256;
+bool prefill_shape_ok(int hidden, int inter);
+cudaError_t launch_split_x(const Dev& d, const float* x, int T, cudaStream_t s);
+cudaError_t launch_prefill_gateup(const Dev& d, int layer, int wave, cudaStream_t s);
+cudaError_t launch_prefill_down(const Dev& d, int layer, int wave, cudaStream_t s);
 
 }  // namespace mf
