@@ -288,13 +288,82 @@ def run_mawforge(args):
         "wall_s": round(wall, 3),
     }
     line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps  # + one reset kernel per step
+    mf.mf_destroy(ctx)
+    if not args.no_prefill:
+        line["prefill"] = prefill_measurement(torch, mf, synth, device)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
-    mf.mf_destroy(ctx)
     if rank == 0:
         print(json.dumps(line))
     if ws > 1:
         torch.distributed.destroy_process_group()
+
+
+def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: float = 15.0) -> dict:
+    """The tensor-core grouped GEMM path on one layer of the 48-layer Q4_0 workload: one
+    4096-token prefill call (Zipf 1.2 routing) from a cold cache, `calls` times after one warm-up.
+    Per call: the GEMM kernels' summed CUDA-event time (gate/up+SwiGLU and down, every wave) and the
+    whole call.  FLOPs: useful = 2 * T * k * 3 * hidden * inter; issued on the tensor cores = 3x that
+    (hi*hi + hi*lo + lo*hi bf16 products)."""
+    cfg = synth.CONFIGS["l48e128q4"]
+    H, E, k, I, q, T = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype, cfg.prefill
+    model = mf.Model(1, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(cache_pct, 1 << 62, 0, 0, T, 0))
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    try:
+        buf = np.empty(plan.payload_bytes, np.uint8)
+        for e in range(E):
+            synth.payload(cfg.model_seed, 0, e, H, I, q, out=buf)
+            mf.mf_pack_put(ctx, 0, e, buf)
+        route = cfg.route_classes[0]
+        x = torch.from_numpy(synth.activations(0, 0, 0, 0, T, H)).to(device)
+        b = torch.from_numpy(synth.plant_bias(synth.routes(0, 0, 0, E, k, T, route.zipf_s, route.reuse), E)).to(device)
+        wr = torch.from_numpy(synth.router_weights(cfg.model_seed, 0, E, H)).to(device)
+        y = torch.empty(T, H, device=device)
+        stream = torch.cuda.Stream(device)
+        gemm_ms, call_ms, mat_ms, n_gemm = [], [], [], 0
+        for i in range(calls + 1):
+            mf.mf_reset(ctx, 0, stream)
+            mf.mf_timing(ctx, ["materialize", "prefill_gemm"])
+            a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                a.record(stream)
+                mf.mf_moe_forward(ctx, 0, x, wr, b, T, y, None, None, stream)
+                z.record(stream)
+            z.synchronize()
+            tm = mf.mf_timing_read(ctx)
+            if i > 0:
+                gemm_ms.append(tm["prefill_gemm"][0])
+                mat_ms.append(tm["materialize"][0])
+                n_gemm = tm["prefill_gemm"][1]
+                call_ms.append(a.elapsed_time(z))
+        mf.mf_timing(ctx, [])
+        assert mf.mf_check(ctx) == 0
+        st = mf.mf_stats(ctx, -1)
+    finally:
+        mf.mf_destroy(ctx)
+    g, c, m = statistics.mean(gemm_ms), statistics.mean(call_ms), statistics.mean(mat_ms)
+    useful = 2.0 * T * k * 3 * H * I
+    issued = 3 * useful
+    peak = _bf16_peak()
+    return {"workload": f"l48e128q4 layer 0: 4096-token prefill call, hidden {H}, {E} experts, top-{k}, inter {I}, "
+                        f"Q4_0, Zipf 1.2, cache {cache_pct:g}% ({plan.slots_per_layer} slots), cold",
+            "tokens_per_s": round(T / (c * 1e-3), 1), "call_ms": round(c, 4), "gemm_ms": round(g, 4),
+            "gemm_waves": n_gemm, "materialize_ms": round(m, 4),
+            "materialize_gbs": round(st["bytes_materialized"] / (m * 1e-3) / 1e9, 1),
+            "useful_tflops": round(useful / (g * 1e-3) / 1e12, 2),
+            "roofline": {"bound": "tensor", "kernel": "prefill grouped GEMMs (gate/up+SwiGLU, down)",
+                         "achieved": round(issued / (g * 1e-3) / 1e12, 2), "peak": peak[0], "unit": "TFLOP/s",
+                         "frac": round(issued / (g * 1e-3) / 1e12 / peak[0], 4), "peak_kind": peak[1],
+                         "flops_per_call": {"useful": useful, "issued": issued}}}
+
+
+def _bf16_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured (burst)"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 def cpu_baseline(n_tokens: int) -> dict:
@@ -355,6 +424,7 @@ def main():
     ap.add_argument("--impl", default="mawforge", choices=["mawforge", "reference"])
     ap.add_argument("--cpu-tokens", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true", help="skip the 4096-token prefill measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle

@@ -134,14 +134,18 @@ int mf_moe_forward(mf_ctx_t* ctx, int layer, const float* x, const float* router
                    const float* logit_bias, int T, float* y, int32_t* idx_out, float* w_out,
                    void* stream);
 
-/* Calls of mf_moe_forward with T >= min_tokens (default 256) run each wave's expert FFN as
- * tcgen05 grouped GEMMs (section "Native Serving Path"'s expert FFN, batched over the tokens
- * each expert serves, as for a prefill chunk): per (expert, 128 assignments, 128 weight rows)
- * the dequantised Q8_0 / Q4_0 weights and the activations, each split into bf16 hi + lo, are
+/* Calls of mf_moe_forward with T >= min_tokens run each wave's expert FFN as tcgen05 grouped
+ * GEMMs (section "Native Serving Path"'s expert FFN, batched over the tokens each expert
+ * serves, as for a prefill chunk): per (expert, 128 assignments, 128 weight rows) the
+ * dequantised Q8_0 / Q4_0 weights and the activations, each split into bf16 hi + lo, are
  * multiplied on the tensor cores with fp32 accumulation (hi*hi + hi*lo + lo*hi).  Smaller T
- * use the dequantising GEMV kernels.  min_tokens = 0 disables the GEMM path; otherwise it
- * must be >= 2, the plan's max_tokens >= 2 and hidden and inter multiples of 128
- * (MF_E_INVAL otherwise).  Host only; applies to calls issued afterwards. */
+ * use the dequantising GEMV kernels.  The default is 256 when the plan's max_tokens >= 256,
+ * else 0 (off).  min_tokens = 0 disables the GEMM path; otherwise it must be >= 2, the plan's
+ * max_tokens >= 2 and hidden and inter multiples of 128 (MF_E_INVAL otherwise).  Enabling it
+ * on a context created with max_tokens < 256 allocates its operand tiles here:
+ * (T k / 128 + min(E, T k)) * 128 * (hidden + inter) * 4 bytes for T = max_tokens (MF_E_OOM
+ * if that fails; MF_E_CUDA if the driver cannot describe the slot pool to the copy engine).
+ * Host only; applies to calls issued afterwards. */
 int mf_prefill_threshold(mf_ctx_t* ctx, int min_tokens);
 
 /* As mf_moe_forward, with x, logit_bias, y, idx_out and w_out in HOST memory (pinned

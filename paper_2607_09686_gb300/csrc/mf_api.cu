@@ -87,7 +87,7 @@ struct Carve {
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
   uint64_t logits, ticket, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
-  uint64_t work, err, xs, sx, sb, sy, sidx, sw;
+  uint64_t work, err, tb_off, sx, sb, sy, sidx, sw;
   uint64_t total;
 };
 
@@ -120,7 +120,7 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.part = c.take<float>(Tm > 1 ? (uint64_t)Tm * k * H : 1);
   o.work = c.take<unsigned>(4);
   o.err = c.take<unsigned>(1);
-  o.xs = c.take<uint16_t>(Tm > 1 ? 2ull * Tm * H : 1);
+  o.tb_off = c.take<int32_t>(E + 1);
   o.sx = c.take<float>((uint64_t)Tm * H);
   o.sb = c.take<float>((uint64_t)Tm * E);
   o.sy = c.take<float>((uint64_t)Tm * H);
@@ -130,10 +130,32 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   return o;
 }
 
+// the tensor-core path's operand tiles are allocated with the context when max_tokens reaches
+// the default threshold (else on first enabling it)
+bool gemm_at_create(const mf_model_t& m, int Tm) { return Tm >= kPrefillMinTokens && prefill_shape_ok(m.hidden, m.inter); }
+
 uint64_t overhead_bytes(const mf_model_t& m, int S, int Tm) {
   const Layout lay = make_layout(m);
   const uint64_t padding = (uint64_t)m.n_layers * S * (lay.stride - lay.canonical);
-  return scratch_layout(m, S, Tm).total + padding;
+  const uint64_t gemm =
+      gemm_at_create(m, Tm) ? prefill_scratch_bytes(Tm, m.top_k, m.n_experts, m.hidden, m.inter) : 0;
+  return scratch_layout(m, S, Tm).total + padding + gemm;
+}
+
+int alloc_gemm_scratch(mf_ctx* c) {
+  if (c->gemm_scratch) return MF_OK;
+  Dev& d = c->d;
+  const uint64_t tiles = prefill_tiles_max(d.T_max, d.k, d.E);
+  uint8_t* p = nullptr;
+  cudaError_t e = cudaMalloc((void**)&p, prefill_scratch_bytes(d.T_max, d.k, d.E, d.H, d.I));
+  if (e != cudaSuccess) {
+    cuda_fail(e, "cudaMalloc(GEMM tiles)");
+    return MF_E_OOM;
+  }
+  c->gemm_scratch = p;
+  d.xt = p;
+  d.ht = p + tiles * (uint64_t)128 * d.H * 4;
+  return MF_OK;
 }
 
 // ---- per-kernel event timing
@@ -178,6 +200,7 @@ void free_ctx(mf_ctx* c) {
   if (c->side) cudaStreamDestroy(c->side);
   if (c->d.slot_of) cudaFree(c->d.slot_of);  // base of the scratch allocation
   if (c->d.pool) cudaFree(c->d.pool);
+  if (c->gemm_scratch) cudaFree(c->gemm_scratch);
   if (c->pack_host) cudaFreeHost(c->pack_host);
   free(c->put_map);
   delete c;
@@ -368,10 +391,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.part = reinterpret_cast<float*>(base + so.part);
   d.work = reinterpret_cast<unsigned*>(base + so.work);
   d.err = reinterpret_cast<unsigned*>(base + so.err);
-  if (Tm > 1) {
-    d.xh = reinterpret_cast<uint16_t*>(base + so.xs);
-    d.xl = d.xh + (size_t)Tm * d.H;
-  }
+  d.tb_off = reinterpret_cast<int32_t*>(base + so.tb_off);
   c->stage_x = reinterpret_cast<float*>(base + so.sx);
   c->stage_bias = reinterpret_cast<float*>(base + so.sb);
   c->stage_y = reinterpret_cast<float*>(base + so.sy);
@@ -411,7 +431,15 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
     return MF_E_INVAL;
   }
   c->decode_pipe = decode_pipe_ok(d) && getenv("MF_DECODE_SIMPLE") == nullptr;
-  c->prefill_min_t = Tm > 1 && prefill_shape_ok(d.H, d.I) ? kPrefillMinTokens : 0;
+  c->tmaps_ok = prefill_shape_ok(d.H, d.I) && prefill_tensor_maps(c) == 0;
+  c->prefill_min_t = 0;
+  if (c->tmaps_ok && gemm_at_create(*m, Tm)) {
+    if ((rc = alloc_gemm_scratch(c)) != MF_OK) {
+      free_ctx(c);
+      return rc;
+    }
+    c->prefill_min_t = kPrefillMinTokens;
+  }
   *out = c;
   return MF_OK;
 }
@@ -475,7 +503,7 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   }
 
   const bool gemm = T > 1 && c->prefill_min_t > 0 && T >= c->prefill_min_t;
-  if (gemm) MF_CUDA(launch_split_x(d, x, T, s));
+  if (gemm) MF_CUDA(launch_tile_x(d, x, T, s));
 
   long long accesses_max = (long long)T * d.k;
   if (accesses_max > d.E) accesses_max = d.E;
@@ -492,8 +520,8 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
     MF_CUDA(cudaStreamWaitEvent(s, c->ev_join[w], 0));
     if (gemm) {
       timer_mark(c, kTPrefill, 0, s);
-      MF_CUDA(launch_prefill_gateup(d, layer, w, s));
-      MF_CUDA(launch_prefill_down(d, layer, w, s));
+      MF_CUDA(launch_prefill_gateup(d, c->tm_gu, layer, w, s));
+      MF_CUDA(launch_prefill_down(d, c->tm_d, layer, w, s));
       timer_mark(c, kTPrefill, 1, s);
       if (w == n_waves - 1) {
         timer_mark(c, kTDown, 0, s);
@@ -527,6 +555,13 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
 int mf_prefill_threshold(mf_ctx_t* c, int min_tokens) {
   if (!c || min_tokens < 0 || min_tokens == 1) return MF_E_INVAL;
   if (min_tokens > 0 && (c->d.T_max < 2 || !prefill_shape_ok(c->d.H, c->d.I))) return MF_E_INVAL;
+  if (min_tokens > 0) {
+    if (!c->tmaps_ok) return MF_E_CUDA;
+    DevGuard guard(c->device);
+    if (!guard.ok) return cuda_fail(cudaSetDevice(c->device), "cudaSetDevice");
+    const int rc = alloc_gemm_scratch(c);
+    if (rc) return rc;
+  }
   c->prefill_min_t = min_tokens;
   return MF_OK;
 }

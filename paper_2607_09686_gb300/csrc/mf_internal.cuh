@@ -1,6 +1,7 @@
 // Internal declarations of the GB300 routed-expert library (not part of the C ABI).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -66,8 +67,11 @@ struct Dev {
   int32_t* miss_list;  // [E + S_alloc] unique index of miss m of wave w at w * S_active + m
   float* h;            // [T_max * k][I]  SwiGLU activations
   float* part;         // [T_max * k][H]  per-assignment down outputs (T > 1)
-  uint16_t* xh;        // [T_max][H]    bf16 high part of x (tensor-core prefill path, T_max > 1)
-  uint16_t* xl;        // [T_max][H]    bf16 low part, x - hi
+  int32_t* tb_off;     // [E + 1]       128-assignment blocks before unique expert u (T > 1)
+  // tensor-core path (many tokens per expert): operand tiles in the MMA's shared-memory order,
+  // per 128-assignment block t and K step kk of 32: [bf16 hi 8 KiB | bf16 lo 8 KiB]
+  uint8_t* xt;         // x tiles:  t * (H / 32) + kk
+  uint8_t* ht;         // h tiles:  t * (I / 32) + kk
   unsigned* work;      // [4]           work-queue counters of the pipelined decode kernels
   unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
 };
@@ -151,6 +155,9 @@ struct mf_ctx {
   uint64_t overhead_bytes;
   bool decode_pipe;  // batch-1 calls use the pipelined decode kernels
   int prefill_min_t;  // calls with T >= this use the tensor-core grouped GEMMs (0 = never)
+  uint8_t* gemm_scratch;  // x and h tiles of the tensor-core path (allocated when first enabled)
+  bool tmaps_ok;
+  CUtensorMap tm_gu, tm_d;  // the slot pool's gate/up and down row records as 3-D byte tensors
 };
 
 namespace mf {
@@ -177,8 +184,11 @@ bool decode_pipe_ok(const Dev& d);
 // many tokens per expert: tcgen05 grouped GEMMs (gate/up + SwiGLU, down) per wave
 constexpr int kPrefillMinTokens = 256;
 bool prefill_shape_ok(int hidden, int inter);
-cudaError_t launch_split_x(const Dev& d, const float* x, int T, cudaStream_t s);
-cudaError_t launch_prefill_gateup(const Dev& d, int layer, int wave, cudaStream_t s);
-cudaError_t launch_prefill_down(const Dev& d, int layer, int wave, cudaStream_t s);
+uint64_t prefill_tiles_max(int T, int k, int E);  // bound on the 128-assignment blocks of a call
+uint64_t prefill_scratch_bytes(int T_max, int k, int E, int hidden, int inter);
+int prefill_tensor_maps(mf_ctx* c);  // encode tm_gu / tm_d for the context's pool; 0 on success
+cudaError_t launch_tile_x(const Dev& d, const float* x, int T, cudaStream_t s);
+cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s);
+cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s);
 
 }  // namespace mf

@@ -103,13 +103,12 @@ extern "C" int mf_expert_ffn_noalloc(const mf_model_t* model, const void* expert
   d.g = const_cast<float*>(g);
 
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  cudaError_t e;
   if (decode_pipe_ok(d)) {
-    if ((e = launch_gateup_single(d, 0, x, s)) != cudaSuccess) return MF_E_CUDA;
-    if ((e = launch_down_single_pipe(d, 0, y, s)) != cudaSuccess) return MF_E_CUDA;
+    if (launch_gateup_single(d, 0, x, s) != cudaSuccess) return MF_E_CUDA;
+    if (launch_down_single_pipe(d, 0, y, s) != cudaSuccess) return MF_E_CUDA;
   } else {
-    if ((e = launch_gateup(d, 0, 0, m.top_k, x, s)) != cudaSuccess) return MF_E_CUDA;
-    if ((e = launch_down_single(d, 0, y, s)) != cudaSuccess) return MF_E_CUDA;
+    if (launch_gateup(d, 0, 0, m.top_k, x, s) != cudaSuccess) return MF_E_CUDA;
+    if (launch_down_single(d, 0, y, s) != cudaSuccess) return MF_E_CUDA;
   }
   return MF_OK;
 }

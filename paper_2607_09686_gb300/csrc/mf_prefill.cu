@@ -13,38 +13,65 @@
 // dropped lo*lo term is below 2^-16 of the product.  Per product the relative error is thus
 // a few times 1e-5, far inside the output tolerance, while the tensor cores do the work.
 //
-// Work unit = (expert of the wave, block of 128 assignments, block of 128 weight rows).  One
-// CTA per SM walks the units.  For each 64-wide K chunk all 256 threads dequantise the weight
-// tiles and gather the assignment tiles into one of two shared-memory stages (no-swizzle
-// K-major core-matrix layout); thread 0 then issues the MMAs (M = 128, N = 128, K = 16 each)
-// and commits them to the stage's mbarrier, so filling stage s+1 overlaps the MMAs of stage s.
-// The epilogue (warps 0-3, one TMEM lane = one weight row each) reads the accumulators with
-// tcgen05.ld.  Every wait is bounded and taken by thread 0, which publishes the outcome
-// before the block acts on it; after a wait gives up the block sets the device error word,
-// waits (bounded) for its MMAs and frees its tensor memory before returning.
+// Operand B never needs a gather inside the GEMM: once per call k_tile_x writes x, split, in
+// the MMA's shared-memory order per (128-assignment block, K step of 32) -- 16 KiB tiles that
+// one bulk copy moves -- and the gate/up epilogue writes h the same way for the down GEMM.
+//
+// Work unit = (expert of the wave, block of 128 assignments, block of 128 weight rows); one
+// CTA of 14 warps per SM walks its units as a flat sequence of K steps of 32 (one quantisation
+// block), with warp-specialised roles linked by mbarriers:
+//   producer (1 warp)    per step: one TMA load per weight tensor (the 128 rows' codes of the
+//                        block, from a 3-D tensor map over the slot pool) into a 3-slot raw ring,
+//                        cp.async of the 128 rows' scale words, and one bulk copy of the B tile
+//                        into operand stage s % 4;
+//   converters (8 warps) dequantise the raw codes exactly into the stage's A tiles (hi / lo,
+//                        no-swizzle K-major core-matrix layout): byte -> float by the
+//                        magic-number conversion, times the binary16 scale, split with packed
+//                        bf16x2 conversions;
+//   MMA (1 thread)       issues the step's tcgen05.mma (M = 128, N = 128, K = 16) into one of two
+//                        TMEM accumulators and commits them to the stage's mbarrier;
+//   epilogue (4 warps)   reads a finished accumulator with tcgen05.ld (warp w: TMEM lanes
+//                        32 (w % 4) .. +31) while the MMAs of the next unit use the other one.
+// Every wait is bounded; a wait that gives up sets the block's flag and the device error word,
+// the roles leave their loops, and the block drains its copies and MMAs (bounded) and frees
+// its tensor memory before returning.
 #include <cuda_bf16.h>
 
-#include "mf_internal.cuh"
+#include "mf_dequant.cuh"
 
 namespace mf {
 namespace {
 
-constexpr int kBM = 128, kBN = 128, kBK = 64;
-constexpr int kThreadsP = 256;
-constexpr uint32_t kTileBytes = kBM * kBK * 2;  // one bf16 tile: 128 rows x 64 k
+using dq::f2_add;
+using dq::f2_fma;
+using dq::f2_pack;
+
+constexpr int kBM = 128, kBN = 128, kBK = 32;
+constexpr int kStages = 4;  // operand stages (A + B tiles)
+constexpr int kRaw = 3;     // raw-code ring slots
+constexpr uint32_t kTile = kBM * kBK * 2;  // one bf16 tile: 128 rows x 32 k = 8 KiB
+constexpr uint32_t kBTile = 2 * kTile;     // B hi + lo, one bulk copy
 constexpr uint32_t kWaitLimit = 1u << 26;
 
-// Byte offset of element (row r, k) in a K-major no-swizzle tile of 128 x 64: 8x8 core
+// warp roles of the 448-thread CTA
+constexpr int kConvWarps = 8;  // warps 0-7: dequantise A tiles
+constexpr int kProdWarp = 8;   // warp 8: copies
+constexpr int kMmaWarp = 9;    // warp 9, lane 0: MMA issue
+constexpr int kEpiWarp0 = 10;  // warps 10-13: epilogue; TMEM lane quarter = warp % 4
+constexpr int kThreadsW = 14 * 32;
+static_assert(kEpiWarp0 == kMmaWarp + 1 && kEpiWarp0 + 4 == kThreadsW / 32, "warp roles");
+
+// Byte offset of element (row r, k) in a K-major no-swizzle tile of 128 x 32: 8x8 core
 // matrices of 128 contiguous bytes, K-adjacent core matrices 128 B apart (the descriptor's
-// leading byte offset), 8-row groups 1024 B apart (its stride byte offset).
-__device__ __forceinline__ uint32_t core_off(int r, int k) {
-  return (uint32_t)((r >> 3) * 1024 + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2);
+// leading byte offset), 8-row groups 512 B apart (its stride byte offset).
+__host__ __device__ __forceinline__ uint32_t core_off(int r, int k) {
+  return (uint32_t)((r >> 3) * 512 + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2);
 }
 
 // shared-memory matrix descriptor: start >> 4, LBO >> 4 at bit 16, SBO >> 4 at bit 32,
 // descriptor version 1 at bit 46, no swizzle
 __device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
-  return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)(128u >> 4) << 16) | ((uint64_t)(1024u >> 4) << 32) |
+  return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)(128u >> 4) << 16) | ((uint64_t)(512u >> 4) << 32) |
          ((uint64_t)1 << 46);
 }
 
@@ -67,6 +94,18 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
 // generic-proxy shared-memory writes become visible to the tensor cores' (async proxy) reads
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+// 3-D tiled TMA load of a box at (x, y, z) of `tmap` into shared memory, completing on `bar`
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* tmap, int x, int y, int z, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+      "[%5];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar))
+      : "memory");
+}
+
 // 16 consecutive fp32 accumulator columns of this thread's TMEM lane
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   uint32_t r[16];
@@ -80,50 +119,46 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-__device__ __forceinline__ void split_bf16(float v, __nv_bfloat16& hi, __nv_bfloat16& lo) {
-  hi = __float2bfloat16_rn(v);
-  lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+__device__ __forceinline__ uint32_t bf2_bits(__nv_bfloat162 v) { return *reinterpret_cast<uint32_t*>(&v); }
+
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
 }
 
-// 8 consecutive K values of one row -> a 16-byte chunk of the hi tile and of the lo tile
-__device__ __forceinline__ void store8(unsigned char* hi_tile, unsigned char* lo_tile, uint32_t off, const float* w) {
+// Two values (packed fp32 pair) -> bf16x2 words hi = bf16(v), lo = bf16(v - hi).
+__device__ __forceinline__ void split2(uint64_t w, uint32_t& hi, uint32_t& lo) {
+  uint32_t a, b;
+  asm("mov.b64 {%0, %1}, %2;" : "=r"(a), "=r"(b) : "l"(w));
+  const __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(a), __uint_as_float(b));
+  const float2 hf = __bfloat1622float2(h);
+  const uint64_t r = f2_fma(f2_pack(__float_as_uint(hf.x), __float_as_uint(hf.y)), f2_pack(0xBF800000u, 0xBF800000u), w);
+  uint32_t ra, rb;
+  asm("mov.b64 {%0, %1}, %2;" : "=r"(ra), "=r"(rb) : "l"(r));
+  hi = bf2_bits(h);
+  lo = bf2_bits(__floats2bfloat162_rn(__uint_as_float(ra), __uint_as_float(rb)));
+}
+
+// Eight byte codes c (two words; Q8_0 c = q + 128, Q4_0 nibbles masked to bytes) times the
+// scale dd = (d, d) -> one 16-byte chunk of the hi tile and of the lo tile at `off`.
+template <uint32_t kOffBits>
+__device__ __forceinline__ void dequant8(uint32_t w0, uint32_t w1, uint64_t dd, unsigned char* hi_t,
+                                         unsigned char* lo_t, uint32_t off) {
+  const uint64_t neg = f2_pack(kOffBits | 0x80000000u, kOffBits | 0x80000000u);  // -(2^23 + offset)
+  const uint32_t ws[2] = {w0, w1};
   uint32_t h[4], l[4];
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    __nv_bfloat16 h0, l0, h1, l1;
-    split_bf16(w[2 * i], h0, l0);
-    split_bf16(w[2 * i + 1], h1, l1);
-    h[i] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-    l[i] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+  for (int i = 0; i < 2; ++i) {
+    const uint64_t q01 =
+        f2_add(f2_pack(__byte_perm(ws[i], 0x4B000000u, 0x7650), __byte_perm(ws[i], 0x4B000000u, 0x7651)), neg);
+    const uint64_t q23 =
+        f2_add(f2_pack(__byte_perm(ws[i], 0x4B000000u, 0x7652), __byte_perm(ws[i], 0x4B000000u, 0x7653)), neg);
+    split2(f2_mul(q01, dd), h[2 * i], l[2 * i]);
+    split2(f2_mul(q23, dd), h[2 * i + 1], l[2 * i + 1]);
   }
-  *reinterpret_cast<uint4*>(hi_tile + off) = make_uint4(h[0], h[1], h[2], h[3]);
-  *reinterpret_cast<uint4*>(lo_tile + off) = make_uint4(l[0], l[1], l[2], l[3]);
-}
-
-// Dequantise one 32-weight block of a slot row record (codes + binary16 scale) into row r of
-// the hi / lo tiles at K = kb*32 .. kb*32 + 31 of the 64-wide chunk.
-template <int QT>
-__device__ __forceinline__ void dequant_block(const uint8_t* codes, const __half* scale, unsigned char* hi,
-                                              unsigned char* lo, int r, int kb) {
-  const float d = __half2float(*scale);
-  float w[32];
-  if constexpr (QT == MF_Q8_0) {  // stored as q + 128
-    const uint4 c0 = *reinterpret_cast<const uint4*>(codes), c1 = *reinterpret_cast<const uint4*>(codes + 16);
-    const uint32_t ws[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-#pragma unroll
-    for (int i = 0; i < 32; ++i) w[i] = d * (float)((int)((ws[i >> 2] >> (8 * (i & 3))) & 0xFF) - 128);
-  } else {  // byte j: element j in the low nibble, element j + 16 in the high nibble
-    const uint4 c = *reinterpret_cast<const uint4*>(codes);
-    const uint32_t ws[4] = {c.x, c.y, c.z, c.w};
-#pragma unroll
-    for (int j = 0; j < 16; ++j) {
-      const uint32_t b = (ws[j >> 2] >> (8 * (j & 3))) & 0xFF;
-      w[j] = d * (float)((int)(b & 0xF) - 8);
-      w[j + 16] = d * (float)((int)(b >> 4) - 8);
-    }
-  }
-#pragma unroll
-  for (int q = 0; q < 4; ++q) store8(hi, lo, core_off(r, kb * 32 + q * 8), w + q * 8);
+  *reinterpret_cast<uint4*>(hi_t + off) = make_uint4(h[0], h[1], h[2], h[3]);
+  *reinterpret_cast<uint4*>(lo_t + off) = make_uint4(l[0], l[1], l[2], l[3]);
 }
 
 struct Unit {
@@ -134,7 +169,7 @@ struct Unit {
 
 // The wave's units, expert by expert: expert u0 + e has ceil(n / 128) assignment blocks times
 // `nrb` row blocks, row blocks innermost (CTAs working on the same assignment block at once
-// share its gathered activations in L2).
+// share its B tiles in L2).
 struct UnitMap {
   int u0, nu, nrb, total;
   const int* pre;  // [nu + 1] exclusive prefix of the experts' unit counts
@@ -150,331 +185,328 @@ struct UnitMap {
   }
 };
 
-__device__ __forceinline__ UnitMap build_units(const Dev& d, int wave, int nrb, int* s_pre) {
-  const int U = d.info[0], S = d.S_active;
-  UnitMap m;
-  m.u0 = wave * S;
-  m.nu = max(0, min(S, U - m.u0));
-  m.nrb = nrb;
-  m.pre = s_pre;
-  if (threadIdx.x == 0) {
-    int acc = 0;
-    for (int e = 0; e < m.nu; ++e) {
-      s_pre[e] = acc;
-      const int n = d.asg_off[m.u0 + e + 1] - d.asg_off[m.u0 + e];
-      acc += (n + kBN - 1) / kBN * nrb;
-    }
-    s_pre[m.nu] = acc;
-  }
-  __syncthreads();
-  m.total = s_pre[m.nu];
-  return m;
-}
-
-// Shared memory: two stages of [NA weight tiles | 2 activation tiles], then the barriers,
-// the assignment of each accumulator column, the unit prefix, the TMEM base and a flag.
-struct PSmem {
-  unsigned char* stage[2];
-  uint64_t* mma_done;   // [2] the MMAs reading stage s have completed
-  uint64_t* acc_ready;  // [1] every MMA issued so far has completed
-  int* pos;             // [kBN] assignment t*k+j of each accumulator column, -1 past the end
-  int* pre;             // [kMaxExperts + 1]
-  uint32_t* tmem;       // [1]
-  int* flag;            // [1] nonzero once a wait gave up
+// Shared memory of one CTA: operand stages, raw ring, barriers, unit prefix.
+template <int NT, int CB>  // tensors per step (2: gate and up, 1: down), code bytes per 32-weight block
+struct PLayout {
+  static constexpr int kNA = 2 * NT;                              // A tiles per stage: hi / lo per tensor
+  static constexpr uint32_t kStage = kNA * kTile + kBTile;        // + B hi / lo
+  static constexpr uint32_t kRawCodes = NT * kBM * CB;            // codes of one step (TMA boxes)
+  static constexpr uint32_t kRawSlot = kRawCodes + NT * kBM * 4;  // + one scale word per (tensor, row)
+  static constexpr int kBars = 2 * kRaw + 2 * kStages + 2 * 2 + 1;
+  static constexpr uint32_t kOffRaw = kStages * kStage;
+  static constexpr uint32_t kOffBar = kOffRaw + kRaw * kRawSlot;
+  static constexpr uint32_t kOffPre = kOffBar + kBars * 8;
+  static constexpr uint32_t kOffMisc = kOffPre + (kMaxExperts + 1) * 4;
+  static constexpr uint32_t kBytes = kOffMisc + 16;
+  static_assert(kRawSlot % 128 == 0 && kOffRaw % 128 == 0, "TMA destinations are 128-byte aligned");
 };
 
-template <int NA>
-__host__ __device__ constexpr uint32_t stage_bytes() {
-  return (NA + 2) * kTileBytes;
-}
+// Gate/up (NT = 2) or down (NT = 1) projection of wave `wave` for every assignment of the wave.
+//   gate/up: A = gate / up rows of the slot's gate/up region, B = x tiles; epilogue
+//            h = silu(G) * U, split, into the h tiles
+//   down:    A = down rows, B = h tiles; epilogue part[assignment][hidden]
+// Pipeline (mbarriers): producer --full--> converters --a_ready--> MMA --mma_done--> producer
+// (B slot) and converters (A slot); converters --raw_free--> producer; MMA --acc_full-->
+// epilogue --acc_empty--> MMA, with two TMEM accumulators.
+template <int QT, int NT>
+__global__ void __launch_bounds__(kThreadsW, 1)
+    k_prefill(const __grid_constant__ CUtensorMap tmap, Dev d, int layer, int wave) {
+  constexpr int CB = QT == MF_Q8_0 ? 32 : 16;
+  using PL = PLayout<NT, CB>;
+  constexpr uint32_t kAcc = NT * kBN;  // TMEM columns of one accumulator (gate | up, or down)
+  constexpr uint32_t kCols = 2 * kAcc;
+  constexpr uint32_t kOffBits = QT == MF_Q8_0 ? dq::kOffQ8 : dq::kOffQ4;
+  extern __shared__ __align__(1024) unsigned char smem[];
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + PL::kOffBar);
+  uint64_t* full = bars;                    // [kRaw]    32 cp.async arrivals + 1 expect-tx arrival
+  uint64_t* raw_free = full + kRaw;         // [kRaw]    one arrival per converter warp
+  uint64_t* a_ready = raw_free + kRaw;      // [kStages] one arrival per converter warp
+  uint64_t* mma_done = a_ready + kStages;   // [kStages] tcgen05.commit
+  uint64_t* acc_full = mma_done + kStages;  // [2]       tcgen05.commit
+  uint64_t* acc_empty = acc_full + 2;       // [2]       one arrival per epilogue warp
+  uint64_t* drain = acc_empty + 2;          // [1]       tcgen05.commit
+  int* s_pre = reinterpret_cast<int*>(smem + PL::kOffPre);
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + PL::kOffMisc);
+  volatile int* s_flag = reinterpret_cast<volatile int*>(smem + PL::kOffMisc + 4);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-template <int NA>
-constexpr size_t prefill_smem() {
-  return 2 * (size_t)stage_bytes<NA>() + 3 * sizeof(uint64_t) + kBN * sizeof(int) + (kMaxExperts + 1) * sizeof(int) +
-         2 * sizeof(uint32_t);
-}
+  const int K = NT == 2 ? d.H : d.I;            // reduction length
+  const int nk = K / kBK;                       // steps per unit
+  const int nrb = (NT == 2 ? d.I : d.H) / kBM;  // row blocks per expert
 
-template <int NA>
-__device__ __forceinline__ PSmem carve_p(unsigned char* base) {
-  PSmem s;
-  s.stage[0] = base;
-  s.stage[1] = base + stage_bytes<NA>();
-  unsigned char* p = base + 2 * stage_bytes<NA>();
-  s.mma_done = reinterpret_cast<uint64_t*>(p);
-  s.acc_ready = s.mma_done + 2;
-  s.pos = reinterpret_cast<int*>(s.acc_ready + 1);
-  s.pre = s.pos + kBN;
-  s.tmem = reinterpret_cast<uint32_t*>(s.pre + kMaxExperts + 1);
-  s.flag = reinterpret_cast<int*>(s.tmem + 1);
-  return s;
-}
-
-// Thread 0 waits (bounded) for the phase of `bar` with the given parity; the whole block then
-// learns the outcome.  Returns false once any wait of the block has given up.
-__device__ __forceinline__ bool block_wait(uint64_t* bar, uint32_t parity, const PSmem& sm, unsigned* err,
-                                           unsigned code) {
-  if (threadIdx.x == 0 && !*sm.flag && !mbar_wait(bar, parity, kWaitLimit)) {
-    *sm.flag = 1;
-    atomicExch(err, code);
+  // ---- prologue: barriers, tensor memory, the wave's unit prefix
+  if (tid == 0) {
+    for (int i = 0; i < kRaw; ++i) {
+      mbar_init(&full[i], 33);
+      mbar_init(&raw_free[i], kConvWarps);
+    }
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&a_ready[i], kConvWarps);
+      mbar_init(&mma_done[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&acc_full[i], 1);
+      mbar_init(&acc_empty[i], 4);
+    }
+    mbar_init(drain, 1);
+    *s_flag = 0;
+    mbar_fence_init();
   }
-  __syncthreads();
-  return *reinterpret_cast<volatile int*>(sm.flag) == 0;
-}
-
-template <uint32_t kCols>
-__device__ __forceinline__ void tmem_alloc(const PSmem& sm) {
-  if (threadIdx.x < 32) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(sm.tmem)),
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(s_tmem)),
                  "r"(kCols));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
-}
-template <uint32_t kCols>
-__device__ __forceinline__ void tmem_free(uint32_t taddr) {
-  if (threadIdx.x < 32) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(kCols));
-}
-
-// Barriers, flag and tensor memory at kernel start.
-template <uint32_t kCols>
-__device__ __forceinline__ uint32_t prologue(const PSmem& sm) {
-  if (threadIdx.x == 0) {
-    mbar_init(&sm.mma_done[0], 1);
-    mbar_init(&sm.mma_done[1], 1);
-    mbar_init(sm.acc_ready, 1);
-    *sm.flag = 0;
-    mbar_fence_init();
-  }
-  tmem_alloc<kCols>(sm);
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  return *sm.tmem;
-}
-
-// At kernel end: wait (bounded) until no MMA is in flight, then free the tensor memory.
-template <uint32_t kCols>
-__device__ __forceinline__ void epilogue_free(const PSmem& sm, uint32_t taddr, uint32_t n_acc, unsigned* err) {
-  if (threadIdx.x == 0) {
-    mma_commit(sm.acc_ready);
-    if (!mbar_wait(sm.acc_ready, n_acc & 1, kWaitLimit)) atomicExch(err, 7u);
+  UnitMap um;
+  um.u0 = wave * d.S_active;
+  um.nu = max(0, min(d.S_active, d.info[0] - um.u0));
+  um.nrb = nrb;
+  um.pre = s_pre;
+  if (tid == 32) {
+    int acc = 0;
+    for (int e = 0; e < um.nu; ++e) {
+      s_pre[e] = acc;
+      acc += (d.tb_off[um.u0 + e + 1] - d.tb_off[um.u0 + e]) * nrb;
+    }
+    s_pre[um.nu] = acc;
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  tmem_free<kCols>(taddr);
-}
+  const uint32_t tmem0 = *s_tmem;
+  um.total = s_pre[um.nu];
+  const int bid = (int)blockIdx.x, nb = (int)gridDim.x;
+  const int n_units = um.total > bid ? (um.total - 1 - bid) / nb + 1 : 0;
+  const int n_steps = n_units * nk;
 
-// Gather the unit's activation rows (bf16 hi/lo [rows][ld]; row = assignment / kdiv) for K
-// chunk c into the B tiles; columns past the unit's n assignments are zero.  Lanes 0-7 of
-// each group of eight take eight consecutive columns, so each 16-byte store of a warp quarter
-// covers all 32 banks.  With `record`, also notes each column's assignment.
-__device__ __forceinline__ void gather_bf16(const uint16_t* __restrict__ src_hi, const uint16_t* __restrict__ src_lo,
-                                            int ld, int kdiv, const int32_t* __restrict__ asg, int a0, int n, int c,
-                                            unsigned char* bhi, unsigned char* blo, int* pos, bool record) {
-  for (int i = threadIdx.x; i < kBN * 8; i += kThreadsP) {
-    const int col = (i & 7) | ((i >> 6) << 3), g = (i >> 3) & 7;
-    uint4 vh = make_uint4(0, 0, 0, 0), vl = make_uint4(0, 0, 0, 0);
-    int p = -1;
-    if (col < n) {
-      p = asg[a0 + col];
-      const size_t off = (size_t)(p / kdiv) * ld + c * kBK + g * 8;
-      vh = *reinterpret_cast<const uint4*>(src_hi + off);
-      vl = *reinterpret_cast<const uint4*>(src_lo + off);
-    }
-    if (record && g == 0) pos[col] = p;
-    *reinterpret_cast<uint4*>(bhi + core_off(col, g * 8)) = vh;
-    *reinterpret_cast<uint4*>(blo + core_off(col, g * 8)) = vl;
-  }
-}
+  // bounded wait; false (and the block's flag and the device error word set) once any wait gave up
+  auto wait = [&](uint64_t* bar, uint32_t parity, unsigned code) -> bool {
+    if (*s_flag) return false;
+    if (mbar_wait(bar, parity, kWaitLimit)) return true;
+    *s_flag = 1;
+    atomicExch(d.err, code);
+    return false;
+  };
 
-// Same from an fp32 [rows][ld] matrix indexed by assignment (the SwiGLU output h), split on
-// the fly.
-__device__ __forceinline__ void gather_f32(const float* __restrict__ src, int ld, const int32_t* __restrict__ asg,
-                                           int a0, int n, int c, unsigned char* bhi, unsigned char* blo, int* pos,
-                                           bool record) {
-  for (int i = threadIdx.x; i < kBN * 8; i += kThreadsP) {
-    const int col = (i & 7) | ((i >> 6) << 3), g = (i >> 3) & 7;
-    float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    int p = -1;
-    if (col < n) {
-      p = asg[a0 + col];
-      const float4* s = reinterpret_cast<const float4*>(src + (size_t)p * ld + c * kBK + g * 8);
-      const float4 f0 = s[0], f1 = s[1];
-      v[0] = f0.x, v[1] = f0.y, v[2] = f0.z, v[3] = f0.w;
-      v[4] = f1.x, v[5] = f1.y, v[6] = f1.z, v[7] = f1.w;
-    }
-    if (record && g == 0) pos[col] = p;
-    store8(bhi, blo, core_off(col, g * 8), v);
-  }
-}
-
-// ---------------------------------------------------------------- gate/up GEMM + SwiGLU
-// h[p][r] = silu(sum_c Wg[r,c] x[p/k][c]) * sum_c Wu[r,c] x[p/k][c] for the wave's assignments
-template <int QT>
-__global__ void __launch_bounds__(kThreadsP, 1) k_prefill_gateup(Dev d, int layer, int wave) {
-  extern __shared__ __align__(1024) unsigned char smem[];
-  const PSmem sm = carve_p<4>(smem);  // weights: gate hi, gate lo, up hi, up lo; then x hi, x lo
-  const uint32_t taddr = prologue<256>(sm);  // columns 0..127 gate, 128..255 up
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const UnitMap um = build_units(d, wave, d.I / kBM, sm.pre);
-  const int nchunk = d.H / kBK;
-  constexpr int kCodeBytes = QT == MF_Q8_0 ? 32 : 16;  // per 32-weight block
-  uint32_t gc = 0, n_acc = 0;                           // chunks filled, accumulator commits
-  for (int ui = blockIdx.x; ui < um.total; ui += gridDim.x) {
-    const Unit un = um.at(ui);
-    const uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[un.u]) * d.lay.stride;
-    const int a0 = d.asg_off[un.u] + un.tb * kBN;
-    const int n = min(kBN, d.asg_off[un.u + 1] - a0);
-    bool ok = true;
-    for (int c = 0; c < nchunk; ++c, ++gc) {
-      const int st_i = (int)(gc & 1);
-      unsigned char* st = sm.stage[st_i];
-      // the MMAs that last read this stage (two chunks ago) must be done before it is refilled
-      if (gc >= 2 && !(ok = block_wait(&sm.mma_done[st_i], ((gc >> 1) - 1) & 1, sm, d.err, 5u))) break;
-      for (int t = threadIdx.x; t < kBM * 4; t += kThreadsP) {  // (row, 32-block, tensor)
-        const int r = t >> 2, kb = (t >> 1) & 1, ten = t & 1;
-        const uint8_t* rec = slot + (size_t)(un.rb * kBM + r) * d.lay.rs_gu;
-        const int blk = c * 2 + kb;
-        const uint8_t* codes = rec + (ten ? d.lay.o_up : 0u) + (size_t)blk * kCodeBytes;
-        const __half* sc = reinterpret_cast<const __half*>(rec + (ten ? d.lay.o_us : d.lay.o_gs)) + blk;
-        dequant_block<QT>(codes, sc, st + (2 * ten) * kTileBytes, st + (2 * ten + 1) * kTileBytes, r, kb);
+  if (warp < kConvWarps) {
+    // ================= converters: raw codes of step s -> A tiles of stage s % kStages
+    // gate/up: thread = (tensor, row), 32 weights; down: thread = (half, row), 16 weights
+    const int r = tid & (kBM - 1), part = tid >> 7;
+    const int ten = NT == 2 ? part : 0, tr = ten * kBM + r;
+    constexpr int kGroups = NT == 2 ? 4 : 2;  // 8-weight groups of this thread
+    const int g0 = NT == 2 ? 0 : part * 2;
+    int kk = 0, slot = 0, stage = 0;
+    uint32_t rph = 0, sph = 0;  // phase parities of the raw ring and of the stage ring
+    for (int s = 0; s < n_steps; ++s) {
+      if (!wait(&full[slot], rph, 1u)) break;
+      if (s >= kStages && !wait(&mma_done[stage], sph ^ 1, 2u)) break;
+      const unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
+      unsigned char* a_hi = smem + stage * PL::kStage + (2 * ten) * kTile;
+      unsigned char* a_lo = a_hi + kTile;
+      const uint32_t sw = *reinterpret_cast<const uint32_t*>(raw + PL::kRawCodes + tr * 4);
+      const float dsc = __half2float(__ushort_as_half((unsigned short)((kk & 1) ? (sw >> 16) : (sw & 0xFFFFu))));
+      const uint64_t dd = f2_pack(__float_as_uint(dsc), __float_as_uint(dsc));
+      const unsigned char* codes = raw + (size_t)tr * CB;
+      if constexpr (QT == MF_Q8_0) {
+#pragma unroll
+        for (int g = 0; g < kGroups; ++g) {
+          const uint2 w = *reinterpret_cast<const uint2*>(codes + (g0 + g) * 8);
+          dequant8<kOffBits>(w.x, w.y, dd, a_hi, a_lo, core_off(r, (g0 + g) * 8));
+        }
+      } else {
+        // byte j: element j (low nibble), element j + 16 (high nibble): groups 0 and 1 are the
+        // low nibbles of bytes 0-7 and 8-15, groups 2 and 3 their high nibbles
+        const uint4 c = *reinterpret_cast<const uint4*>(codes);
+        const uint32_t ws[4] = {c.x, c.y, c.z, c.w};
+#pragma unroll
+        for (int g = 0; g < kGroups; ++g) {
+          const int gg = g0 + g;
+          const int sh = gg >= 2 ? 4 : 0, wb = (gg & 1) * 2;
+          dequant8<kOffBits>((ws[wb] >> sh) & 0x0F0F0F0Fu, (ws[wb + 1] >> sh) & 0x0F0F0F0Fu, dd, a_hi, a_lo,
+                             core_off(r, gg * 8));
+        }
       }
-      gather_bf16(d.xh, d.xl, d.H, d.k, d.asg, a0, n, c, st + 4 * kTileBytes, st + 5 * kTileBytes, sm.pos, c == 0);
-      fence_async_smem();
-      __syncthreads();
-      if (threadIdx.x == 0) {
+      fence_async_smem();  // this thread's A writes, before the MMAs read them
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&a_ready[stage]);
+        mbar_arrive(&raw_free[slot]);
+      }
+      if (++kk == nk) kk = 0;
+      if (++slot == kRaw) slot = 0, rph ^= 1;
+      if (++stage == kStages) stage = 0, sph ^= 1;
+    }
+  } else if (warp == kProdWarp) {
+    // ================= producer: TMA boxes of codes, cp.async of scale words, bulk B tile
+    const size_t rstride = NT == 2 ? d.lay.rs_gu : d.lay.rs_d;
+    const uint8_t* tiles = NT == 2 ? d.xt : d.ht;
+    const uint8_t* rows = nullptr;  // the unit's first weight row record
+    int y0 = 0, z0 = 0;             // its TMA coordinates: first row, slot plane
+    size_t b0 = 0;                  // its first B tile
+    int kk = 0, slot = 0, stage = 0, j = 0;
+    uint32_t rph = 0, sph = 0;
+    constexpr uint32_t kTx = NT * kBM * CB + kBTile;
+    for (int s = 0; s < n_steps; ++s) {
+      if (kk == 0) {
+        const Unit un = um.at(bid + j * nb);
+        z0 = layer * d.S_alloc + d.uslot[un.u];
+        y0 = un.rb * kBM;
+        rows = d.pool + (size_t)z0 * d.lay.stride + (NT == 2 ? 0 : d.lay.d_off) + (size_t)y0 * rstride;
+        b0 = (size_t)(d.tb_off[un.u] + un.tb) * nk;
+      }
+      if (s >= kRaw && !wait(&raw_free[slot], rph ^ 1, 3u)) break;
+      if (s >= kStages && !wait(&mma_done[stage], sph ^ 1, 4u)) break;
+      unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
+      if (lane == 0) {
+        mbar_arrive_tx(&full[slot], kTx);
+#pragma unroll
+        for (int tn = 0; tn < NT; ++tn)
+          tma_load_3d(raw + tn * kBM * CB, &tmap, (tn ? (int)d.lay.o_up : 0) + kk * CB, y0, z0, &full[slot]);
+        bulk_g2s(smem + stage * PL::kStage + PL::kNA * kTile, tiles + (b0 + kk) * kBTile, kBTile, &full[slot]);
+      }
+#pragma unroll
+      for (int i = 0; i < NT * kBM / 32; ++i) {
+        const int t = lane + 32 * i, tn = t / kBM, r = t % kBM;
+        const uint32_t so = NT == 2 ? (tn ? d.lay.o_us : d.lay.o_gs) : d.lay.o_ds;
+        cp_async4(raw + PL::kRawCodes + t * 4, rows + (size_t)r * rstride + so + (size_t)(kk & ~1) * 2);
+      }
+      asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&full[slot])) : "memory");
+      if (++kk == nk) kk = 0, ++j;
+      if (++slot == kRaw) slot = 0, rph ^= 1;
+      if (++stage == kStages) stage = 0, sph ^= 1;
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
+  } else if (warp == kMmaWarp) {
+    // ================= MMA issue (one thread)
+    if (lane == 0) {
+      int kk = 0, stage = 0, j = 0;
+      uint32_t sph = 0;
+      for (int s = 0; s < n_steps; ++s) {
+        const uint32_t acc = tmem0 + (uint32_t)(j & 1) * kAcc;
+        if (kk == 0 && j >= 2 && !wait(&acc_empty[j & 1], ((j >> 1) - 1) & 1, 8u)) break;
+        if (!wait(&a_ready[stage], sph, 9u)) break;
         tc_fence_after();
-        const uint32_t base = smem_u32(st);
+        const uint32_t base = smem_u32(smem + stage * PL::kStage);
+        const uint64_t bh = smem_desc(base + PL::kNA * kTile), bl = smem_desc(base + PL::kNA * kTile + kTile);
 #pragma unroll
         for (int ks = 0; ks < kBK / 16; ++ks) {
-          const uint32_t ko = ks * 256;  // K = 16 spans two core matrices
-          const uint64_t bh = smem_desc(base + 4 * kTileBytes + ko), bl = smem_desc(base + 5 * kTileBytes + ko);
+          const uint64_t ko = (ks * 256) >> 4;  // K = 16 spans two core matrices
 #pragma unroll
-          for (int ten = 0; ten < 2; ++ten) {
-            const uint64_t ah = smem_desc(base + (2 * ten) * kTileBytes + ko);
-            const uint64_t al = smem_desc(base + (2 * ten + 1) * kTileBytes + ko);
-            const uint32_t dt = taddr + ten * kBN;
-            mma_bf16(dt, ah, bh, (c | ks) != 0);
-            mma_bf16(dt, ah, bl, 1);
-            mma_bf16(dt, al, bh, 1);
+          for (int tn = 0; tn < NT; ++tn) {
+            const uint64_t ah = smem_desc(base + (2 * tn) * kTile) + ko;
+            const uint64_t al = smem_desc(base + (2 * tn + 1) * kTile) + ko;
+            const uint32_t dt = acc + tn * kBN;
+            mma_bf16(dt, ah, bh + ko, (kk | ks) != 0);
+            mma_bf16(dt, ah, bl + ko, 1);
+            mma_bf16(dt, al, bh + ko, 1);
           }
         }
-        mma_commit(&sm.mma_done[st_i]);
+        mma_commit(&mma_done[stage]);
+        if (kk == nk - 1) mma_commit(&acc_full[j & 1]);
+        if (++kk == nk) kk = 0, ++j;
+        if (++stage == kStages) stage = 0, sph ^= 1;
       }
+      // nothing may be in flight when the tensor memory is freed
+      mma_commit(drain);
+      if (!mbar_wait(drain, 0, kWaitLimit)) atomicExch(d.err, 10u);
     }
-    if (!ok) break;
-    // every MMA of the unit done -> h = silu(gate) * up
-    if (threadIdx.x == 0) mma_commit(sm.acc_ready);
-    if (!block_wait(sm.acc_ready, n_acc & 1, sm, d.err, 6u)) break;
-    ++n_acc;
-    tc_fence_after();
-    if (warp < 4) {
-      const int r = un.rb * kBM + warp * 32 + lane;
-      const uint32_t lane_addr = taddr + ((uint32_t)(warp * 32) << 16);
-      for (int c0 = 0; c0 < n; c0 += 16) {
-        float g[16], u[16];
-        tmem_ld16(lane_addr + c0, g);
-        tmem_ld16(lane_addr + kBN + c0, u);
+  } else {
+    // ================= epilogue: accumulator j & 1 -> outputs
+    const int q4 = warp & 3;  // TMEM lanes 32 q4 .. 32 q4 + 31 = weight rows of the block
+    for (int j = 0; j < n_units; ++j) {
+      if (!wait(&acc_full[j & 1], (j >> 1) & 1, 11u)) break;
+      tc_fence_after();
+      const Unit un = um.at(bid + j * nb);
+      const int a0 = d.asg_off[un.u] + un.tb * kBN;
+      const int n = min(kBN, d.asg_off[un.u + 1] - a0);
+      const int r = un.rb * kBM + q4 * 32 + lane;  // weight row = output feature
+      const uint32_t lane_addr = tmem0 + (uint32_t)(j & 1) * kAcc + ((uint32_t)(q4 * 32) << 16);
+      if constexpr (NT == 2) {
+        // h tile of K step r / 32 of the down GEMM: this lane's row is its k = r % 32
+        uint8_t* ht = d.ht + ((size_t)(d.tb_off[un.u] + un.tb) * (d.I / kBK) + (r >> 5)) * kBTile;
+        for (int c0 = 0; c0 < kBN; c0 += 16) {
+          float g[16], u[16];
+          tmem_ld16(lane_addr + c0, g);
+          tmem_ld16(lane_addr + kBN + c0, u);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int p = sm.pos[c0 + j];
-          if (p >= 0) d.h[(size_t)p * d.I + r] = g[j] / (1.0f + expf(-g[j])) * u[j];
+          for (int q = 0; q < 16; ++q) {
+            const int col = c0 + q;
+            const float hv = col < n ? g[q] / (1.0f + expf(-g[q])) * u[q] : 0.0f;
+            const __nv_bfloat16 hi = __float2bfloat16_rn(hv);
+            const uint32_t o = core_off(col, r & 31);
+            *reinterpret_cast<uint16_t*>(ht + o) = __bfloat16_as_ushort(hi);
+            *reinterpret_cast<uint16_t*>(ht + kTile + o) =
+                __bfloat16_as_ushort(__float2bfloat16_rn(hv - __bfloat162float(hi)));
+          }
+        }
+      } else {
+        for (int c0 = 0; c0 < n; c0 += 32) {
+          const int pl = c0 + lane < n ? __ldg(&d.asg[a0 + c0 + lane]) : -1;  // assignment of column c0 + lane
+#pragma unroll
+          for (int hlf = 0; hlf < 2; ++hlf) {
+            if (c0 + hlf * 16 >= n) break;
+            float v[16];
+            tmem_ld16(lane_addr + c0 + hlf * 16, v);
+#pragma unroll
+            for (int q = 0; q < 16; ++q) {
+              const int p = __shfl_sync(0xffffffffu, pl, hlf * 16 + q);
+              if (p >= 0) d.part[(size_t)p * d.H + r] = v[q];
+            }
+          }
         }
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acc_empty[j & 1]);
     }
-    tc_fence_before();
-    __syncthreads();  // accumulators read before the next unit's first MMA overwrites them
   }
-  epilogue_free<256>(sm, taddr, n_acc, d.err);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem0), "r"(kCols));
 }
 
-// ---------------------------------------------------------------- down GEMM
-// part[p][c] = sum_r Wd[c,r] h[p][r] for the wave's assignments
-template <int QT>
-__global__ void __launch_bounds__(kThreadsP, 1) k_prefill_down(Dev d, int layer, int wave) {
-  extern __shared__ __align__(1024) unsigned char smem[];
-  const PSmem sm = carve_p<2>(smem);  // weights: down hi, down lo; then h hi, h lo
-  const uint32_t taddr = prologue<128>(sm);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const UnitMap um = build_units(d, wave, d.H / kBM, sm.pre);
-  const int nchunk = d.I / kBK;
-  constexpr int kCodeBytes = QT == MF_Q8_0 ? 32 : 16;
-  uint32_t gc = 0, n_acc = 0;
-  for (int ui = blockIdx.x; ui < um.total; ui += gridDim.x) {
-    const Unit un = um.at(ui);
-    const uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[un.u]) * d.lay.stride + d.lay.d_off;
-    const int a0 = d.asg_off[un.u] + un.tb * kBN;
-    const int n = min(kBN, d.asg_off[un.u + 1] - a0);
-    bool ok = true;
-    for (int c = 0; c < nchunk; ++c, ++gc) {
-      const int st_i = (int)(gc & 1);
-      unsigned char* st = sm.stage[st_i];
-      if (gc >= 2 && !(ok = block_wait(&sm.mma_done[st_i], ((gc >> 1) - 1) & 1, sm, d.err, 5u))) break;
-      for (int t = threadIdx.x; t < kBM * 2; t += kThreadsP) {  // (row, 32-block)
-        const int r = t >> 1, kb = t & 1;
-        const uint8_t* rec = slot + (size_t)(un.rb * kBM + r) * d.lay.rs_d;
-        const int blk = c * 2 + kb;
-        dequant_block<QT>(rec + (size_t)blk * kCodeBytes, reinterpret_cast<const __half*>(rec + d.lay.o_ds) + blk, st,
-                          st + kTileBytes, r, kb);
-      }
-      gather_f32(d.h, d.I, d.asg, a0, n, c, st + 2 * kTileBytes, st + 3 * kTileBytes, sm.pos, c == 0);
-      fence_async_smem();
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        tc_fence_after();
-        const uint32_t base = smem_u32(st);
-#pragma unroll
-        for (int ks = 0; ks < kBK / 16; ++ks) {
-          const uint32_t ko = ks * 256;
-          const uint64_t ah = smem_desc(base + ko), al = smem_desc(base + kTileBytes + ko);
-          const uint64_t bh = smem_desc(base + 2 * kTileBytes + ko), bl = smem_desc(base + 3 * kTileBytes + ko);
-          mma_bf16(taddr, ah, bh, (c | ks) != 0);
-          mma_bf16(taddr, ah, bl, 1);
-          mma_bf16(taddr, al, bh, 1);
-        }
-        mma_commit(&sm.mma_done[st_i]);
-      }
+// x (fp32 [T][H]) -> the x tiles of every 128-assignment block of the call: block t (of unique
+// expert u, assignments asg_off[u] + 128 tb ..), K step kk: column c = assignment, row k,
+// split into bf16 hi and lo; columns past the expert's assignments are zero.
+__global__ void __launch_bounds__(256) k_tile_x(Dev d, const float* __restrict__ x) {
+  __shared__ int s_row[kBN];
+  __shared__ int s_u, s_tb;
+  const int t = blockIdx.x;
+  const int U = d.info[0];
+  if (t >= d.tb_off[U]) return;
+  if (threadIdx.x == 0) {
+    int lo = 0, hi = U - 1;
+    while (lo < hi) {  // last expert with tb_off[u] <= t
+      const int mid = (lo + hi + 1) >> 1;
+      if (d.tb_off[mid] <= t) lo = mid;
+      else hi = mid - 1;
     }
-    if (!ok) break;
-    if (threadIdx.x == 0) mma_commit(sm.acc_ready);
-    if (!block_wait(sm.acc_ready, n_acc & 1, sm, d.err, 6u)) break;
-    ++n_acc;
-    tc_fence_after();
-    if (warp < 4) {
-      const int r = un.rb * kBM + warp * 32 + lane;  // output feature
-      const uint32_t lane_addr = taddr + ((uint32_t)(warp * 32) << 16);
-      for (int c0 = 0; c0 < n; c0 += 16) {
-        float v[16];
-        tmem_ld16(lane_addr + c0, v);
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int p = sm.pos[c0 + j];
-          if (p >= 0) d.part[(size_t)p * d.H + r] = v[j];
-        }
-      }
-    }
-    tc_fence_before();
-    __syncthreads();
+    s_u = lo;
+    s_tb = t - d.tb_off[lo];
   }
-  epilogue_free<128>(sm, taddr, n_acc, d.err);
-}
-
-// x (fp32 [T][H]) -> bf16 hi and lo parts, once per call
-__global__ void k_split_x(const float4* __restrict__ x, size_t n4, uint2* __restrict__ hi, uint2* __restrict__ lo) {
-  for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n4; i += (size_t)gridDim.x * blockDim.x) {
-    const float4 v = x[i];
-    const float f[4] = {v.x, v.y, v.z, v.w};
-    uint32_t h[2], l[2];
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      __nv_bfloat16 h0, l0, h1, l1;
-      split_bf16(f[2 * q], h0, l0);
-      split_bf16(f[2 * q + 1], h1, l1);
-      h[q] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-      l[q] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+  __syncthreads();
+  const int a0 = d.asg_off[s_u] + s_tb * kBN, n = min(kBN, d.asg_off[s_u + 1] - a0);
+  for (int c = threadIdx.x; c < kBN; c += blockDim.x) s_row[c] = c < n ? d.asg[a0 + c] / d.k : -1;
+  __syncthreads();
+  const int nk = d.H / kBK;
+  uint8_t* tile0 = d.xt + (size_t)t * nk * kBTile;
+  // item i = (column i >> 2, 8-value group i & 3) of one K step: 512 per step
+  for (int it = threadIdx.x; it < nk * 512; it += blockDim.x) {
+    const int kk = it >> 9, i = it & 511, col = i >> 2, g = i & 3;
+    uint32_t h[4] = {0, 0, 0, 0}, l[4] = {0, 0, 0, 0};
+    const int row = s_row[col];
+    if (row >= 0) {
+      const float4* src = reinterpret_cast<const float4*>(x + (size_t)row * d.H + kk * kBK + g * 8);
+      const float4 v0 = __ldg(src), v1 = __ldg(src + 1);
+      split2(f2_pack(__float_as_uint(v0.x), __float_as_uint(v0.y)), h[0], l[0]);
+      split2(f2_pack(__float_as_uint(v0.z), __float_as_uint(v0.w)), h[1], l[1]);
+      split2(f2_pack(__float_as_uint(v1.x), __float_as_uint(v1.y)), h[2], l[2]);
+      split2(f2_pack(__float_as_uint(v1.z), __float_as_uint(v1.w)), h[3], l[3]);
     }
-    hi[i] = make_uint2(h[0], h[1]);
-    lo[i] = make_uint2(l[0], l[1]);
+    uint8_t* tile = tile0 + (size_t)kk * kBTile + core_off(col, g * 8);
+    *reinterpret_cast<uint4*>(tile) = make_uint4(h[0], h[1], h[2], h[3]);
+    *reinterpret_cast<uint4*>(tile + kTile) = make_uint4(l[0], l[1], l[2], l[3]);
   }
 }
 
@@ -489,33 +521,78 @@ int sm_count_p() {
   return n;
 }
 
-template <class K>
-cudaError_t launch_persistent(K kernel, size_t smem, const Dev& d, int layer, int wave, cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+template <int QT, int NT>
+cudaError_t launch_k(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s) {
+  constexpr size_t smem = PLayout<NT, QT == MF_Q8_0 ? 32 : 16>::kBytes;
+  static_assert(smem <= 232448, "shared memory per block");
+  cudaError_t e = cudaFuncSetAttribute(k_prefill<QT, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  kernel<<<sm_count_p(), kThreadsP, smem, s>>>(d, layer, wave);
+  k_prefill<QT, NT><<<sm_count_p(), kThreadsW, smem, s>>>(tm, d, layer, wave);
   return cudaGetLastError();
+}
+
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// One region of every slot as a 3-D byte tensor: (byte in row record, row, slot plane).
+int encode_region(EncodeTiled enc, CUtensorMap* tm, void* base, uint64_t rec_bytes, uint64_t rows, uint64_t planes,
+                  uint64_t plane_stride, uint32_t box_bytes) {
+  const cuuint64_t dims[3] = {rec_bytes, rows, planes};
+  const cuuint64_t strides[2] = {rec_bytes, plane_stride};
+  const cuuint32_t box[3] = {box_bytes, (cuuint32_t)kBM, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, base, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+                 CUDA_SUCCESS
+             ? 0
+             : -1;
 }
 
 }  // namespace
 
+// shapes the GEMM path serves: whole 128-row blocks in both projections (which also makes the
+// scale words read in pairs lie inside each row's scales)
 bool prefill_shape_ok(int H, int I) { return H > 0 && I > 0 && H % kBM == 0 && I % kBM == 0; }
 
-cudaError_t launch_split_x(const Dev& d, const float* x, int T, cudaStream_t s) {
-  const size_t n4 = (size_t)T * d.H / 4;
-  k_split_x<<<2 * sm_count_p(), 256, 0, s>>>(reinterpret_cast<const float4*>(x), n4, reinterpret_cast<uint2*>(d.xh),
-                                             reinterpret_cast<uint2*>(d.xl));
+// Each unique expert adds at most one partial block: sum_u ceil(n_u / 128) <= T k / 128 + min(E, T k).
+uint64_t prefill_tiles_max(int T, int k, int E) {
+  const uint64_t a = (uint64_t)T * k;
+  return a / kBN + (a < (uint64_t)E ? a : (uint64_t)E);
+}
+
+uint64_t prefill_scratch_bytes(int T_max, int k, int E, int H, int I) {
+  return prefill_tiles_max(T_max, k, E) * (uint64_t)kBN * (uint64_t)(H + I) * 4;  // hi + lo bf16
+}
+
+int prefill_tensor_maps(mf_ctx* c) {
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || !fn)
+    return -1;
+  const EncodeTiled enc = reinterpret_cast<EncodeTiled>(fn);
+  const Dev& d = c->d;
+  const uint32_t cb = d.qtype == MF_Q8_0 ? 32 : 16;
+  const uint64_t planes = (uint64_t)d.L * d.S_alloc;
+  if (encode_region(enc, &c->tm_gu, d.pool, d.lay.rs_gu, (uint64_t)d.I, planes, d.lay.stride, cb)) return -1;
+  if (encode_region(enc, &c->tm_d, d.pool + d.lay.d_off, d.lay.rs_d, (uint64_t)d.H, planes, d.lay.stride, cb))
+    return -1;
+  return 0;
+}
+
+cudaError_t launch_tile_x(const Dev& d, const float* x, int T, cudaStream_t s) {
+  const uint64_t blocks = prefill_tiles_max(T, d.k, d.E);
+  k_tile_x<<<(unsigned)blocks, 256, 0, s>>>(d, x);
   return cudaGetLastError();
 }
 
-cudaError_t launch_prefill_gateup(const Dev& d, int layer, int wave, cudaStream_t s) {
-  return d.qtype == MF_Q8_0 ? launch_persistent(k_prefill_gateup<MF_Q8_0>, prefill_smem<4>(), d, layer, wave, s)
-                            : launch_persistent(k_prefill_gateup<MF_Q4_0>, prefill_smem<4>(), d, layer, wave, s);
+cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s) {
+  return d.qtype == MF_Q8_0 ? launch_k<MF_Q8_0, 2>(d, tm, layer, wave, s) : launch_k<MF_Q4_0, 2>(d, tm, layer, wave, s);
 }
 
-cudaError_t launch_prefill_down(const Dev& d, int layer, int wave, cudaStream_t s) {
-  return d.qtype == MF_Q8_0 ? launch_persistent(k_prefill_down<MF_Q8_0>, prefill_smem<2>(), d, layer, wave, s)
-                            : launch_persistent(k_prefill_down<MF_Q4_0>, prefill_smem<2>(), d, layer, wave, s);
+cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s) {
+  return d.qtype == MF_Q8_0 ? launch_k<MF_Q8_0, 1>(d, tm, layer, wave, s) : launch_k<MF_Q4_0, 1>(d, tm, layer, wave, s);
 }
 
 }  // namespace mf

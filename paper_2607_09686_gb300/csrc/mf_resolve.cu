@@ -78,6 +78,12 @@ __global__ void __launch_bounds__(256) k_resolve(Dev d, int layer, int T) {
       acc += cnt[s_uniq[u]];
     }
     d.asg_off[U] = acc;
+    int tiles = 0;  // 128-assignment blocks before each expert's (the grouped GEMMs' tile index)
+    for (int u = 0; u < U; ++u) {
+      d.tb_off[u] = tiles;
+      tiles += (cnt[s_uniq[u]] + 127) / 128;
+    }
+    d.tb_off[U] = tiles;
   }
   __syncthreads();
   for (int p = tid; p < n; p += nt) {
