@@ -28,7 +28,8 @@
 //                        no-swizzle K-major core-matrix layout): byte -> float by the
 //                        magic-number conversion, times the binary16 scale, split with packed
 //                        bf16x2 conversions;
-//   MMA (1 thread)       issues the step's tcgen05.mma (M = 128, N = 128, K = 16) into one of two
+//   MMA (1 thread)       issues the step's tcgen05.mma (M = 128, K = 16, N = the block's assignments
+//                        rounded up to a multiple of 16) into one of two
 //                        TMEM accumulators and commits them to the stage's mbarrier;
 //   epilogue (4 warps)   reads a finished accumulator with tcgen05.ld (warp w: TMEM lanes
 //                        32 (w % 4) .. +31) while the MMAs of the next unit use the other one.
@@ -75,14 +76,18 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
          ((uint64_t)1 << 46);
 }
 
-// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, both K-major, M x N
-constexpr uint32_t kIdesc =
-    (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+// kind::f16 instruction descriptor: fp32 accumulator, bf16 A and B, both K-major, M = 128 x N
+// (N a multiple of 16, at most 128 here)
+__device__ __forceinline__ uint32_t idesc_n(int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
+// the MMA width of a block with n assignments: n rounded up to a multiple of 16
+__device__ __forceinline__ int n_eff(int n) { return max(16, (n + 15) & ~15); }
 
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accumulate) {
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
   asm volatile(
       "{ .reg .pred p; setp.ne.u32 p, %4, 0; tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(d_tmem),
-      "l"(a), "l"(b), "r"(kIdesc), "r"(accumulate));
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
 }
 // arrive on `bar` once every MMA this thread issued so far has completed
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
@@ -287,6 +292,8 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     atomicExch(d.err, code);
     return false;
   };
+  // the same for a whole warp: lane 0 polls, the warp synchronises and shares the outcome
+  auto warp_wait = [&](uint64_t* bar, uint32_t parity, unsigned code) -> bool { return wait(bar, parity, code); };
 
   if (warp < kConvWarps) {
     // ================= converters: raw codes of step s -> A tiles of stage s % kStages
@@ -298,8 +305,8 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     int kk = 0, slot = 0, stage = 0;
     uint32_t rph = 0, sph = 0;  // phase parities of the raw ring and of the stage ring
     for (int s = 0; s < n_steps; ++s) {
-      if (!wait(&full[slot], rph, 1u)) break;
-      if (s >= kStages && !wait(&mma_done[stage], sph ^ 1, 2u)) break;
+      if (!warp_wait(&full[slot], rph, 1u)) break;
+      if (s >= kStages && !warp_wait(&mma_done[stage], sph ^ 1, 2u)) break;
       const unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
       unsigned char* a_hi = smem + stage * PL::kStage + (2 * ten) * kTile;
       unsigned char* a_lo = a_hi + kTile;
@@ -343,9 +350,9 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     const uint8_t* rows = nullptr;  // the unit's first weight row record
     int y0 = 0, z0 = 0;             // its TMA coordinates: first row, slot plane
     size_t b0 = 0;                  // its first B tile
+    uint32_t b_bytes = 0;           // bytes of each B half the MMAs read: n_eff columns
     int kk = 0, slot = 0, stage = 0, j = 0;
     uint32_t rph = 0, sph = 0;
-    constexpr uint32_t kTx = NT * kBM * CB + kBTile;
     for (int s = 0; s < n_steps; ++s) {
       if (kk == 0) {
         const Unit un = um.at(bid + j * nb);
@@ -353,16 +360,21 @@ __global__ void __launch_bounds__(kThreadsW, 1)
         y0 = un.rb * kBM;
         rows = d.pool + (size_t)z0 * d.lay.stride + (NT == 2 ? 0 : d.lay.d_off) + (size_t)y0 * rstride;
         b0 = (size_t)(d.tb_off[un.u] + un.tb) * nk;
+        const int a0 = d.asg_off[un.u] + un.tb * kBN;
+        b_bytes = (uint32_t)n_eff(min(kBN, d.asg_off[un.u + 1] - a0)) * (kBK * 2);
       }
-      if (s >= kRaw && !wait(&raw_free[slot], rph ^ 1, 3u)) break;
-      if (s >= kStages && !wait(&mma_done[stage], sph ^ 1, 4u)) break;
+      if (s >= kRaw && !warp_wait(&raw_free[slot], rph ^ 1, 3u)) break;
+      if (s >= kStages && !warp_wait(&mma_done[stage], sph ^ 1, 4u)) break;
       unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
       if (lane == 0) {
-        mbar_arrive_tx(&full[slot], kTx);
+        mbar_arrive_tx(&full[slot], NT * kBM * CB + 2 * b_bytes);
 #pragma unroll
         for (int tn = 0; tn < NT; ++tn)
           tma_load_3d(raw + tn * kBM * CB, &tmap, (tn ? (int)d.lay.o_up : 0) + kk * CB, y0, z0, &full[slot]);
-        bulk_g2s(smem + stage * PL::kStage + PL::kNA * kTile, tiles + (b0 + kk) * kBTile, kBTile, &full[slot]);
+        unsigned char* bdst = smem + stage * PL::kStage + PL::kNA * kTile;
+        const uint8_t* bsrc = tiles + (b0 + kk) * kBTile;
+        bulk_g2s(bdst, bsrc, b_bytes, &full[slot]);                  // hi: the first n_eff columns
+        bulk_g2s(bdst + kTile, bsrc + kTile, b_bytes, &full[slot]);  // lo
       }
 #pragma unroll
       for (int i = 0; i < NT * kBM / 32; ++i) {
@@ -380,9 +392,14 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     // ================= MMA issue (one thread)
     if (lane == 0) {
       int kk = 0, stage = 0, j = 0;
-      uint32_t sph = 0;
+      uint32_t sph = 0, idesc = 0;
       for (int s = 0; s < n_steps; ++s) {
         const uint32_t acc = tmem0 + (uint32_t)(j & 1) * kAcc;
+        if (kk == 0) {
+          const Unit un = um.at(bid + j * nb);
+          const int a0 = d.asg_off[un.u] + un.tb * kBN;
+          idesc = idesc_n(n_eff(min(kBN, d.asg_off[un.u + 1] - a0)));
+        }
         if (kk == 0 && j >= 2 && !wait(&acc_empty[j & 1], ((j >> 1) - 1) & 1, 8u)) break;
         if (!wait(&a_ready[stage], sph, 9u)) break;
         tc_fence_after();
@@ -396,9 +413,9 @@ __global__ void __launch_bounds__(kThreadsW, 1)
             const uint64_t ah = smem_desc(base + (2 * tn) * kTile) + ko;
             const uint64_t al = smem_desc(base + (2 * tn + 1) * kTile) + ko;
             const uint32_t dt = acc + tn * kBN;
-            mma_bf16(dt, ah, bh + ko, (kk | ks) != 0);
-            mma_bf16(dt, ah, bl + ko, 1);
-            mma_bf16(dt, al, bh + ko, 1);
+            mma_bf16(dt, ah, bh + ko, idesc, (kk | ks) != 0);
+            mma_bf16(dt, ah, bl + ko, idesc, 1);
+            mma_bf16(dt, al, bh + ko, idesc, 1);
           }
         }
         mma_commit(&mma_done[stage]);
@@ -414,7 +431,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     // ================= epilogue: accumulator j & 1 -> outputs
     const int q4 = warp & 3;  // TMEM lanes 32 q4 .. 32 q4 + 31 = weight rows of the block
     for (int j = 0; j < n_units; ++j) {
-      if (!wait(&acc_full[j & 1], (j >> 1) & 1, 11u)) break;
+      if (!warp_wait(&acc_full[j & 1], (j >> 1) & 1, 11u)) break;
       tc_fence_after();
       const Unit un = um.at(bid + j * nb);
       const int a0 = d.asg_off[un.u] + un.tb * kBN;
@@ -424,7 +441,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
       if constexpr (NT == 2) {
         // h tile of K step r / 32 of the down GEMM: this lane's row is its k = r % 32
         uint8_t* ht = d.ht + ((size_t)(d.tb_off[un.u] + un.tb) * (d.I / kBK) + (r >> 5)) * kBTile;
-        for (int c0 = 0; c0 < kBN; c0 += 16) {
+        for (int c0 = 0; c0 < n_eff(n); c0 += 16) {  // the columns the down MMAs read
           float g[16], u[16];
           tmem_ld16(lane_addr + c0, g);
           tmem_ld16(lane_addr + kBN + c0, u);
