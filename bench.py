@@ -32,20 +32,25 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "l4e64"
 N_TOKENS = 256
 
-# DRAM bytes (read + write) of one gate/up launch from the ncu capture summarised in
-# profiles/k_gateup_pipe_l4e64_decode.md, valid while the kernel sources hash to `sha`.
-GATEUP_TRAFFIC = {"sha": "81f6b54c28f8fe9f", "bytes": 26780672,
+# DRAM bytes (read + write) of one launch of the roofline kernel (the fused one-token FFN) from
+# the ncu capture summarised under profiles/, valid while the kernel sources hash to `sha`
+# (otherwise the line reports null: the counters no longer describe the kernel that ran).
+KERNEL_TRAFFIC = {"sha": None, "bytes": None,
                   "files": ("paper_2607_09686_gb300/csrc/mf_decode.cu", "paper_2607_09686_gb300/csrc/mf_dequant.cuh",
                             "paper_2607_09686_gb300/csrc/mf_internal.cuh")}
 
 
-def _captured_traffic():
+def _sources_sha():
     import hashlib
     h = hashlib.sha256()
-    for f in GATEUP_TRAFFIC["files"]:
+    for f in KERNEL_TRAFFIC["files"]:
         with open(os.path.join(ROOT, f), "rb") as fh:
             h.update(fh.read())
-    return GATEUP_TRAFFIC["bytes"] if h.hexdigest()[:16] == GATEUP_TRAFFIC["sha"] else None
+    return h.hexdigest()[:16]
+
+
+def _captured_traffic():
+    return KERNEL_TRAFFIC["bytes"] if KERNEL_TRAFFIC["sha"] == _sources_sha() else None
 
 
 def _peaks():
@@ -155,30 +160,36 @@ def run_mawforge(args):
             for l in range(L):
                 mf.mf_moe_forward(ctx, l, x[t, l], wr[l], bias[t, l], 1, y[t, l], None, None, stream)
 
-    # one graph per step (the 1024 calls of a 256-token sequence), captured through the C ABI with
-    # the library's per-kernel event records inside, so the kernel times come from the timed replays
-    timed = ["materialize", "gateup_swiglu", "down_combine"]
-    graph = torch.cuda.CUDAGraph()
+    # one graph per step (the 1024 calls of a 256-token sequence), captured through the C ABI.  The
+    # timed steps replay a graph without instrumentation; the per-kernel breakdown comes from the
+    # same calls captured a second time with the library's CUDA-event records around each launch
+    # (graph nodes, so they time the launches of those replays), replayed right after.
+    timed = ["materialize", "ffn_fused", "gateup_swiglu", "down_combine"]
+    graph, graph_k = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
         step_calls()  # untimed eager pass: warms the pool
         stream.synchronize()
-        mf.mf_timing(ctx, timed)
+        mf.mf_timing(ctx, [])
         with torch.cuda.graph(graph, stream=stream):
+            step_calls()
+        mf.mf_timing(ctx, timed)
+        with torch.cuda.graph(graph_k, stream=stream):
             step_calls()
     torch.cuda.synchronize()
 
-    def one_step(ev0, ev1):
+    def one_step(g, ev0, ev1):
         with torch.cuda.stream(stream):
             flush.zero_()
             ev0.record(stream)
-            graph.replay()
+            g.replay()
             ev1.record(stream)
 
     for _ in range(args.warmup):
-        one_step(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+        one_step(graph, torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
     torch.cuda.synchronize()
 
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    evk = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     kt = {name: [0.0, 0] for name in mf.KERNEL_CLASSES}
     if ws > 1:
         torch.distributed.barrier()
@@ -186,14 +197,18 @@ def run_mawforge(args):
     with ClockSampler(local) as clk:
         t0 = time.perf_counter()
         for i in range(args.steps):
-            one_step(*evs[i])
+            one_step(graph, *evs[i])
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+        for i in range(args.steps):  # instrumented replays: kernel breakdown
+            one_step(graph_k, *evk[i])
             for name, (kms, n) in mf.mf_timing_read(ctx).items():  # waits for this replay (outside its events)
                 kt[name][0] += kms
                 kt[name][1] += n
         torch.cuda.synchronize()
-        wall = time.perf_counter() - t0
     step_ms = [a.elapsed_time(b) for a, b in evs]
     ms = sum(step_ms) / len(step_ms)
+    ms_instrumented = sum(a.elapsed_time(b) for a, b in evk) / len(evk)
     if ws > 1:
         t = torch.tensor([ms], device=device)
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
@@ -242,9 +257,18 @@ def run_mawforge(args):
     dn_bytes = k * H * (cfg.inter // 32) * 34 + 4 * k * cfg.inter + 4 * H
     ms_gu, n_gu = kt["gateup_swiglu"]
     ms_dn, n_dn = kt["down_combine"]
+    ms_ff, n_ff = kt["ffn_fused"]
     ms_mat, n_mat = kt["materialize"]
-    gemv_gbs = (gu_bytes * n_gu + dn_bytes * n_dn) / ((ms_gu + ms_dn) * 1e-3) / 1e9
-    gu_gbs = gu_bytes / (ms_gu / n_gu * 1e-3) / 1e9
+    if n_ff:  # one launch per call: gate/up + SwiGLU + down + combine
+        rf_kernel = "ffn_fused (grouped dequant-GEMV: k experts' gate/up rows, then their down rows, one launch)"
+        rf_bytes = gu_bytes + dn_bytes
+        rf_gbs = rf_bytes / (ms_ff / n_ff * 1e-3) / 1e9
+    else:
+        rf_kernel = "gateup_swiglu (grouped dequant-GEMV, k experts' gate+up rows)"
+        rf_bytes = gu_bytes
+        rf_gbs = gu_bytes / (ms_gu / n_gu * 1e-3) / 1e9
+    gemv_ms = ms_ff + ms_gu + ms_dn
+    gemv_gbs = (gu_bytes + dn_bytes) * (n_ff + n_gu) / (gemv_ms * 1e-3) / 1e9
     tokens = N_TOKENS * args.steps * ws
     value = N_TOKENS / (ms * 1e-3) * ws
     clocks = clk.summary()
@@ -258,6 +282,7 @@ def run_mawforge(args):
         "steps": args.steps,
         "warmup": args.warmup,
         "ms_per_step": round(ms, 4),
+        "ms_per_step_instrumented": round(ms_instrumented, 4),
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
@@ -271,12 +296,11 @@ def run_mawforge(args):
         "cache": {"hit_rate": round(st["hits"] / max(1, st["accesses"]), 4),
                   "materialized_bytes_per_token": st["bytes_materialized"] / N_TOKENS,
                   "misses_per_token": st["misses"] / N_TOKENS, "accesses_per_step": st["accesses"]},
-        "roofline": {"bound": "hbm", "kernel": "gateup_swiglu (grouped dequant-GEMV, k experts' gate+up rows)",
-                     "achieved": round(gu_gbs, 1), "peak": hbm, "unit": "GB/s",
-                     "frac": round(gu_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": _captured_traffic(),
-                     "gemv_pair_gbs": round(gemv_gbs, 1), "gemv_pair_frac": round(gemv_gbs / hbm, 4),
-                     "frac_of_8tbs": round(gemv_gbs / 8000.0, 4),
-                     "bytes_per_launch": {"gateup": gu_bytes, "down": dn_bytes}},
+        "roofline": {"bound": "hbm", "kernel": rf_kernel,
+                     "achieved": round(rf_gbs, 1), "peak": hbm, "unit": "GB/s",
+                     "frac": round(rf_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": _captured_traffic(),
+                     "bytes_per_launch": rf_bytes, "frac_of_8tbs": round(gemv_gbs / 8000.0, 4),
+                     "timing": "CUDA events around each launch in instrumented replays of the step graph"},
         "kernels": kernels,
         "copy": {"materialized_bytes_per_step": st["bytes_materialized"],
                  "materialize_gbs": round(args.steps * st["bytes_materialized"] / (ms_mat * 1e-3) / 1e9, 1)
@@ -287,7 +311,9 @@ def run_mawforge(args):
         "gpu_launches": None,
         "wall_s": round(wall, 3),
     }
-    line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps  # + one reset kernel per step
+    # every kernel of the timed replays: the timed classes (counted in the instrumented replays of
+    # the same calls), one router per call and one reset per step
+    line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps * (N_TOKENS * L + 1)
     mf.mf_destroy(ctx)
     if not args.no_prefill:
         line["prefill"] = prefill_measurement(torch, mf, synth, device)

@@ -174,9 +174,10 @@ int mf_trace(mf_ctx_t* ctx, int layer, int32_t* experts, int32_t* slots, uint8_t
 
 /* Per-kernel timing with CUDA events recorded on the stream each kernel runs on.
  * class_mask selects the kernel classes timed (bit i: 0 router, 1 resolve, 2 materialise,
- * 3 gate/up+SwiGLU, 4 down+combine, 5 prefill grouped GEMM; 0 stops timing); each call clears
+ * 3 gate/up+SwiGLU, 4 down+combine, 5 prefill grouped GEMMs, 6 one-token expert FFN (gate/up,
+ * SwiGLU, down and combine in one launch); 0 stops timing); each call clears
  * earlier records.  mf_timing_read synchronises and writes for each class the summed
- * milliseconds and the number of timed launches into ms[6] and launches[6].  Calls captured
+ * milliseconds and the number of timed launches into ms[7] and launches[7].  Calls captured
  * into a CUDA graph while timing is on capture their event records as graph nodes; after each
  * replay mf_timing_read reports that replay. */
 int mf_timing(mf_ctx_t* ctx, unsigned class_mask);

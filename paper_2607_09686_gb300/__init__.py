@@ -24,7 +24,7 @@ __all__ = [
 Q4_0 = 2
 Q8_0 = 8
 MF_OK, MF_E_INVAL, MF_E_BUDGET, MF_E_OOM, MF_E_CUDA, MF_E_STATE, MF_E_TIMEOUT = 0, -1, -2, -3, -4, -5, -6
-KERNEL_CLASSES = ("router", "resolve", "materialize", "gateup_swiglu", "down_combine", "prefill_gemm")
+KERNEL_CLASSES = ("router", "resolve", "materialize", "gateup_swiglu", "down_combine", "prefill_gemm", "ffn_fused")
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmawforge.so")
 if not os.path.exists(LIB_PATH):
@@ -218,10 +218,10 @@ def mf_timing(ctx: int, classes=None) -> None:
 
 def mf_timing_read(ctx: int) -> dict:
     """{kernel class: (summed ms, launches)} from the CUDA events of each launch."""
-    ms = (ctypes.c_double * 6)()
-    n = (ctypes.c_int64 * 6)()
+    ms = (ctypes.c_double * len(KERNEL_CLASSES))()
+    n = (ctypes.c_int64 * len(KERNEL_CLASSES))()
     _check(_lib.mf_timing_read(ctx, ms, n), "mf_timing_read")
-    return {KERNEL_CLASSES[i]: (float(ms[i]), int(n[i])) for i in range(6)}
+    return {KERNEL_CLASSES[i]: (float(ms[i]), int(n[i])) for i in range(len(KERNEL_CLASSES))}
 
 
 def mf_check(ctx: int) -> int:

@@ -431,6 +431,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
     return MF_E_INVAL;
   }
   c->decode_pipe = decode_pipe_ok(d) && getenv("MF_DECODE_SIMPLE") == nullptr;
+  c->ffn_fused = c->decode_pipe && ffn_fused_ok(d) && getenv("MF_DECODE_UNFUSED") == nullptr;
   c->tmaps_ok = prefill_shape_ok(d.H, d.I) && prefill_tensor_maps(c) == 0;
   c->prefill_min_t = 0;
   if (c->tmaps_ok && gemm_at_create(*m, Tm)) {
@@ -528,6 +529,12 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
         MF_CUDA(launch_combine(d, T, y, s));
         timer_mark(c, kTDown, 1, s);
       }
+      continue;
+    }
+    if (T == 1 && c->ffn_fused) {
+      timer_mark(c, kTFfn, 0, s);
+      MF_CUDA(launch_ffn_single(d, layer, x, y, s));
+      timer_mark(c, kTFfn, 1, s);
       continue;
     }
     const bool pipe = T == 1 && c->decode_pipe;

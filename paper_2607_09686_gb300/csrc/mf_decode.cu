@@ -34,6 +34,7 @@ constexpr int kConsumers = 16;
 constexpr int kThreads = (kConsumers + 1) * 32;
 constexpr int kMaxStages = 12;
 constexpr size_t kSmemBudget = 200 * 1024;
+constexpr size_t kFusedSmem = 224 * 1024;  // the fused kernel's dynamic + static shared memory
 
 struct PipeCfg {
   int R;                 // rows per item
@@ -75,9 +76,10 @@ size_t smem_bytes(const PipeCfg& c) {
 
 // The consumers split `n` vectors of kW values into int8 pieces, one vector per thread, into
 // shared memory, then wait for each other (the producer keeps streaming meanwhile).
-template <int QT>
+template <int QT, bool kCoherent = false>
 __device__ __forceinline__ void split_vectors(const float* __restrict__ src, int n, XQ<QT>* dst) {
-  for (int i = threadIdx.x; i < n; i += kConsumers * 32) dst[i] = quant_vec<QT>(src + (size_t)i * Vec<QT>::kW);
+  for (int i = threadIdx.x; i < n; i += kConsumers * 32)
+    dst[i] = quant_vec<QT, kCoherent>(src + (size_t)i * Vec<QT>::kW);
   named_bar_sync(1, kConsumers * 32);
 }
 
@@ -302,6 +304,249 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
   __syncthreads();
 }
 
+// ---------------------------------------------------------------- fused gate/up + down, one token
+// Both projections in one persistent cooperative launch.  A block's down work is a contiguous
+// range of rpc output rows: its item j is expert j's rpc down records, one bulk copy into a buffer
+// of its own.  The producer requests those k copies right after the first gate/up items (the down
+// weights do not depend on h), then streams the rest of the gate/up items through the ring, so the
+// whole call's weights are in flight from the start.  The consumers form h = silu(gate) * up for
+// their gate/up items, publish it, meet every other block at a grid-wide arrival counter (bounded
+// wait), and then take the down items with the k experts' h.  The counter never resets: each launch adds one
+// arrival per block, and a block waits for the multiple of gridDim.x that completes its launch.
+struct FusedCfg {
+  PipeCfg g;
+  int rpc;               // down: output rows per block (a contiguous range)
+  uint32_t dn_bytes;     // down item: one expert's rpc down records (one bulk copy, own buffer)
+  int n_hvec;            // h vectors of the k experts, split into int8 pieces
+  int NS;                // gate/up ring stages
+  uint32_t stage_bytes;  // gate/up item
+  int red_floats;        // partial results: gate/up items x 16 warps, then k x rpc down rows
+  uint32_t vq_bytes;
+  // shared memory: [NS gate/up stages | k down buffers | full | empty | full_d | red | vq]
+  size_t off_dn, off_bar, off_red, off_vq, total;
+};
+
+// The arrival is a release (the block's h, written before it and published to this thread by the
+// block barrier, becomes visible with it); the polling loads acquire.
+__device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, unsigned* err) {
+  unsigned long long old;
+  asm volatile("atom.add.release.gpu.global.u64 %0, [%1], 1;" : "=l"(old) : "l"(arrive) : "memory");
+  const unsigned long long target = (old / gridDim.x + 1) * gridDim.x;
+  for (uint32_t i = 0; i < (1u << 22); ++i) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(arrive) : "memory");
+    if (v >= target) return true;
+    if (i >= 64) __nanosleep(32);
+  }
+  atomicExch(err, 5u);
+  return false;
+}
+
+template <int QT, int VPL, int VPLD>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, float* __restrict__ y, FusedCfg f) {
+  extern __shared__ __align__(128) unsigned char smem[];
+  __shared__ const uint8_t* s_gu[kMaxTopK];
+  __shared__ const uint8_t* s_dn[kMaxTopK];
+  __shared__ float s_g[kMaxTopK];
+  const PipeCfg& cg = f.g;
+  Smem sm;
+  sm.stage0 = smem;
+  sm.full = reinterpret_cast<uint64_t*>(smem + f.off_bar);
+  sm.empty = sm.full + kMaxStages;
+  uint64_t* full_d = sm.empty + kMaxStages;  // [kMaxTopK] down buffers, one use each
+  unsigned char* dbuf = smem + f.off_dn;
+  sm.red = reinterpret_cast<float*>(smem + f.off_red);
+  sm.vq = smem + f.off_vq;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int k = d.k;
+  const int mine_g = items_of_block(cg.n_items);
+  const int r0 = (int)blockIdx.x * f.rpc, nrows = max(0, min(d.H - r0, f.rpc));  // this block's down rows
+  const int mine_d = nrows > 0 ? k : 0;
+  if (threadIdx.x < k) {
+    const uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
+    s_gu[threadIdx.x] = slot;
+    s_dn[threadIdx.x] = slot + d.lay.d_off;
+    s_g[threadIdx.x] = d.g[threadIdx.x];
+  }
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < f.NS; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kConsumers);
+    }
+    for (int j = 0; j < k; ++j) mbar_init(&full_d[j], 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  if (warp == kConsumers) {
+    if (lane == 0) {
+      const int grid = (int)gridDim.x;
+      Ring ring;
+      int it = 0;
+      bool ok = true;
+      // gate/up items: R contiguous row records of expert u; after the first ring's worth (or
+      // two items, whichever is fewer), the k down copies
+      const int R = cg.R, nrb = d.I / R;
+      const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
+      const int first = min(mine_g, min(2, f.NS));
+      int u = (int)blockIdx.x / nrb, rb = (int)blockIdx.x % nrb;
+      bool d_issued = false;
+      for (int i = 0; i < mine_g && ok; ++i, ++it) {
+        if (i == first) {
+          d_issued = true;
+          const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
+          const size_t off = (size_t)r0 * d.lay.rs_d;
+          for (int j = 0; j < mine_d; ++j) {
+            mbar_arrive_tx(&full_d[j], dbytes);
+            bulk_g2s(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + off, dbytes, &full_d[j]);
+          }
+        }
+        if (it >= f.NS && !(ok = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u))) break;
+        uint64_t* bar = &sm.full[ring.s];
+        mbar_arrive_tx(bar, bytes);
+        bulk_g2s(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar);
+        ring.next(f.NS);
+        rb += grid;
+        while (rb >= nrb) {
+          rb -= nrb;
+          ++u;
+        }
+      }
+      if (!d_issued && ok) {  // fewer gate/up items than `first`: the down copies go now
+        const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
+        const size_t off = (size_t)r0 * d.lay.rs_d;
+        for (int j = 0; j < mine_d; ++j) {
+          mbar_arrive_tx(&full_d[j], dbytes);
+          bulk_g2s(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + off, dbytes, &full_d[j]);
+        }
+        d_issued = true;
+      }
+      if (!ok) atomicExch(d.err, 1u);
+      // no copy may be in flight when the block exits: wait for the last use of every stage
+      for (int s = 0; s < f.NS && s < it; ++s) {
+        const int uses = (it - 1 - s) / f.NS + 1;
+        if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u)) atomicExch(d.err, 2u);
+      }
+      if (d_issued)
+        for (int j = 0; j < mine_d; ++j)
+          if (!mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
+    }
+  } else {
+    Ring ring;
+    bool ok = true;
+    // ---- gate/up: warp w: tensor w / (R*cs), row (w / cs) % R, column range w % cs
+    {
+      const int R = cg.R, cs = cg.cs, nrb = d.I / R;
+      const uint32_t rs = d.lay.rs_gu;
+      const int ten = warp / (R * cs), row = (warp / cs) % R, col = warp % cs;
+      const int nv = (d.lay.qrow_gu / 16) / cs;
+      const int v0 = col * nv;
+      const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
+      split_vectors<QT>(x, cg.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq));
+      XQ<QT> xr[VPL];
+#pragma unroll
+      for (int i = 0; i < VPL; ++i) {
+        const int v = lane + 32 * i;
+        if (v < nv) xr[i] = xq[v0 + v];
+      }
+      for (int it = 0; it < mine_g; ++it) {
+        if (!(ok = mbar_wait(&sm.full[ring.s], ring.phase))) break;
+        const unsigned char* rec = sm.stage0 + (size_t)ring.s * f.stage_bytes + row * rs;
+        const unsigned char* q = rec + ten * d.lay.o_up + 16 * v0;
+        const __half* sc = reinterpret_cast<const __half*>(rec + (ten ? d.lay.o_us : d.lay.o_gs));
+        float acc = 0.f;
+#pragma unroll
+        for (int i = 0; i < VPL; ++i) {
+          const int v = lane + 32 * i;
+          if (v < nv)
+            acc = fmaf(dot_q<QT>(*reinterpret_cast<const uint4*>(q + 16 * v), xr[i]),
+                       __half2float(sc[scale_index<QT>(v0 + v)]), acc);
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) sm.red[it * kConsumers + warp] = acc;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&sm.empty[ring.s]);
+        ring.next(f.NS);
+      }
+      named_bar_sync(1, kConsumers * 32);
+      for (int t = threadIdx.x; t < mine_g * R; t += kConsumers * 32) {
+        const int it = t / R, r = t % R;
+        const float* p = sm.red + it * kConsumers;
+        float ag = 0.f, au = 0.f;
+        for (int cc = 0; cc < cs; ++cc) {
+          ag += p[(0 * R + r) * cs + cc];
+          au += p[(1 * R + r) * cs + cc];
+        }
+        const int item = (int)blockIdx.x + it * (int)gridDim.x;
+        d.h[(size_t)(item / nrb) * d.I + (item % nrb) * R + r] = ag / (1.0f + expf(-ag)) * au;
+      }
+      named_bar_sync(1, kConsumers * 32);  // the block's h written
+    }
+    // ---- every block's h published (one arrival per block, always, so launches stay aligned)
+    if (threadIdx.x == 0 && !grid_arrive_wait(reinterpret_cast<unsigned long long*>(d.work), d.err)) ok = false;
+    named_bar_sync(1, kConsumers * 32);
+    // ---- down: warp w holds expert j = w / (16 / k)'s h in registers for the whole phase and
+    // takes rows sub, sub + 16 / k, ... of that expert's item (sub = w % (16 / k))
+    {
+      const int nvec = d.lay.qrow_d / 16;
+      const uint32_t rs = d.lay.rs_d;
+      const XQ<QT>* hq = reinterpret_cast<const XQ<QT>*>(sm.vq);
+      split_vectors<QT, true>(d.h, f.n_hvec, reinterpret_cast<XQ<QT>*>(sm.vq));  // written by other blocks
+      float* red = sm.red + cg.max_mine * kConsumers;  // [k][rpc]
+      const int wpe = kConsumers / k, j = warp / wpe, sub = warp % wpe;
+      if (j < mine_d && ok) {
+        XQ<QT> hr[VPLD];
+#pragma unroll
+        for (int i = 0; i < VPLD; ++i) {
+          const int v = lane + 32 * i;
+          if (v < nvec) hr[i] = hq[j * nvec + v];
+        }
+        if ((ok = mbar_wait(&full_d[j], 0))) {
+          const unsigned char* st = dbuf + (size_t)j * f.dn_bytes;
+          // four rows at a time: independent dot products and interleaved reductions
+          for (int row0 = sub; row0 < nrows; row0 += 4 * wpe) {
+            float acc[4];
+#pragma unroll
+            for (int rr = 0; rr < 4; ++rr) {
+              const int row = row0 + rr * wpe;
+              acc[rr] = 0.f;
+              if (row < nrows) {
+                const unsigned char* q = st + (size_t)row * rs;
+                const __half* sc = reinterpret_cast<const __half*>(q + d.lay.o_ds);
+#pragma unroll
+                for (int i = 0; i < VPLD; ++i) {
+                  const int v = lane + 32 * i;
+                  if (v < nvec)
+                    acc[rr] = fmaf(dot_q<QT>(*reinterpret_cast<const uint4*>(q + 16 * v), hr[i]),
+                                   __half2float(sc[scale_index<QT>(v)]), acc[rr]);
+                }
+              }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+              for (int rr = 0; rr < 4; ++rr) acc[rr] += __shfl_xor_sync(0xffffffffu, acc[rr], o);
+            if (lane == 0)
+#pragma unroll
+              for (int rr = 0; rr < 4; ++rr)
+                if (row0 + rr * wpe < nrows) red[j * f.rpc + row0 + rr * wpe] = acc[rr];
+          }
+        }
+      }
+      if (!ok && lane == 0) atomicExch(d.err, 3u);
+      named_bar_sync(1, kConsumers * 32);
+      // combine the k experts of each row in rank order
+      for (int row = threadIdx.x; row < nrows; row += kConsumers * 32) {
+        float acc = 0.f;
+        for (int jj = 0; jj < k; ++jj) acc = fmaf(s_g[jj], red[jj * f.rpc + row], acc);
+        y[r0 + row] = acc;
+      }
+    }
+  }
+  __syncthreads();
+}
+
 int vpl_for(int nvec) {
   const int need = (nvec + 31) / 32;
   return need <= 1 ? 1 : need <= 2 ? 2 : need <= 3 ? 3 : need <= 4 ? 4 : 8;
@@ -406,6 +651,64 @@ cudaError_t down_pipe_q(const Dev& d, int layer, float* y, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+FusedCfg fused_cfg(const Dev& d) {
+  FusedCfg f;
+  f.g = gateup_cfg(d);
+  f.rpc = (d.H + sm_count() - 1) / sm_count();
+  f.dn_bytes = (uint32_t)f.rpc * d.lay.rs_d;
+  f.n_hvec = d.k * (d.lay.qrow_d / 16);
+  const uint32_t hv_bytes = (uint32_t)(f.n_hvec * (d.qtype == MF_Q8_0 ? sizeof(XQ<kQ8>) : sizeof(XQ<kQ4>)));
+  f.stage_bytes = f.g.stage_bytes;
+  f.red_floats = f.g.max_mine * kConsumers + d.k * f.rpc;
+  f.vq_bytes = f.g.vq_bytes > hv_bytes ? f.g.vq_bytes : hv_bytes;
+  const size_t fixed = (size_t)d.k * f.dn_bytes + (2 * kMaxStages + kMaxTopK) * sizeof(uint64_t) +
+                       (size_t)f.red_floats * sizeof(float) + f.vq_bytes;
+  const size_t budget = kFusedSmem - 1024;  // - the kernel's static shared memory
+  const size_t ns = fixed < budget ? (budget - fixed) / f.stage_bytes : 0;
+  f.NS = (int)(ns > (size_t)kMaxStages ? kMaxStages : ns);
+  f.off_dn = (size_t)f.NS * f.stage_bytes;
+  f.off_bar = f.off_dn + (size_t)d.k * f.dn_bytes;
+  f.off_red = f.off_bar + (2 * kMaxStages + kMaxTopK) * sizeof(uint64_t);
+  f.off_vq = f.off_red + (((size_t)f.red_floats * sizeof(float) + 15) & ~(size_t)15);
+  f.total = f.off_vq + f.vq_bytes;
+  return f;
+}
+
+size_t fused_smem(const FusedCfg& f) { return f.total; }
+
+template <class Kern>
+cudaError_t launch_coop(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x, float* y,
+                        const FusedCfg& f) {
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(sm_count());
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;  // every block resident: they wait for each other
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
+}
+
+template <int QT>
+cudaError_t ffn_pipe_q(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
+  const FusedCfg f = fused_cfg(d);
+  const size_t smem = fused_smem(f);
+  const int vx = vpl_for((d.lay.qrow_gu / 16) / f.g.cs), vh = vpl_for(d.lay.qrow_d / 16);
+#define MF_FF(A, B) \
+  if (vx == A && vh == B) return launch_coop(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, y, f);
+  MF_FF(1, 1) MF_FF(1, 2) MF_FF(2, 1) MF_FF(2, 2)
+  if constexpr (QT == kQ8) {  // Q4_0 takes at most two vectors per lane (decode_pipe_ok)
+    MF_FF(1, 3) MF_FF(2, 3) MF_FF(3, 1) MF_FF(3, 2) MF_FF(3, 3) MF_FF(4, 1) MF_FF(4, 2) MF_FF(4, 3)
+  }
+#undef MF_FF
+  return cudaErrorInvalidConfiguration;
+}
+
 }  // namespace
 
 // The pipelined kernels apply when the register-held vectors fit without spills (Q8_0: at most
@@ -430,5 +733,11 @@ cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStrea
 }
 
 size_t decode_smem_bytes(const Dev& d, int which) { return smem_bytes(which == 0 ? gateup_cfg(d) : down_cfg(d)); }
+
+bool ffn_fused_ok(const Dev& d) { return decode_pipe_ok(d) && fused_cfg(d).NS >= 2; }
+
+cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
+  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, y, s) : ffn_pipe_q<kQ4>(d, layer, x, y, s);
+}
 
 }  // namespace mf

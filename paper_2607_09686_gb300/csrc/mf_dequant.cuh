@@ -114,13 +114,15 @@ struct XQ {
   float sf;     // s / 127^2
 };
 
-template <int QT>
+// kCoherent: read through L2 only (for vectors other blocks of the same kernel wrote)
+template <int QT, bool kCoherent = false>
 __device__ __forceinline__ XQ<QT> quant_vec(const float* __restrict__ vp) {
   constexpr int kW = Vec<QT>::kW;
   float v[kW];
 #pragma unroll
   for (int i = 0; i < kW / 4; ++i) {
-    const float4 f = __ldg(reinterpret_cast<const float4*>(vp) + i);
+    const float4 f =
+        kCoherent ? __ldcg(reinterpret_cast<const float4*>(vp) + i) : __ldg(reinterpret_cast<const float4*>(vp) + i);
     v[4 * i] = f.x;
     v[4 * i + 1] = f.y;
     v[4 * i + 2] = f.z;

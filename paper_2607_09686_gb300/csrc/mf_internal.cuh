@@ -12,8 +12,8 @@ namespace mf {
 
 constexpr int kMaxTopK = 8;
 constexpr int kMaxExperts = 1024;
-constexpr int kTimerClasses = 6;
-enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5 };
+constexpr int kTimerClasses = 7;
+enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5, kTFfn = 6 };
 
 // Layout of one expert slot, identical in the pinned pack and in the HBM pool: row records.
 // Gate/up region: I records, record r = [gate codes row r | up codes row r | gate scales row r
@@ -72,7 +72,7 @@ struct Dev {
   // per 128-assignment block t and K step kk of 32: [bf16 hi 8 KiB | bf16 lo 8 KiB]
   uint8_t* xt;         // x tiles:  t * (H / 32) + kk
   uint8_t* ht;         // h tiles:  t * (I / 32) + kk
-  unsigned* work;      // [4]           work-queue counters of the pipelined decode kernels
+  unsigned* work;      // [4]           arrival counter (64-bit) of the fused one-token FFN kernel
   unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
 };
 
@@ -154,6 +154,7 @@ struct mf_ctx {
   cudaEvent_t* timer_ev[mf::kTimerClasses];  // pairs: [2 * i], [2 * i + 1]
   uint64_t overhead_bytes;
   bool decode_pipe;  // batch-1 calls use the pipelined decode kernels
+  bool ffn_fused;    // ... fused into one cooperative launch
   int prefill_min_t;  // calls with T >= this use the tensor-core grouped GEMMs (0 = never)
   uint8_t* gemm_scratch;  // x and h tiles of the tensor-core path (allocated when first enabled)
   bool tmaps_ok;
@@ -181,6 +182,9 @@ cudaError_t launch_gateup_single(const Dev& d, int layer, const float* x, cudaSt
 cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStream_t s);
 size_t decode_smem_bytes(const Dev& d, int which);
 bool decode_pipe_ok(const Dev& d);
+// both projections of one token in one cooperative launch (d.work holds its arrival counter)
+bool ffn_fused_ok(const Dev& d);
+cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s);
 // many tokens per expert: tcgen05 grouped GEMMs (gate/up + SwiGLU, down) per wave
 constexpr int kPrefillMinTokens = 256;
 bool prefill_shape_ok(int hidden, int inter);

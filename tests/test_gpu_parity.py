@@ -73,20 +73,25 @@ def test_l4e64_decode(pct):
     _decode_run(Shape.of(cfg), S, cfg.n_tokens, seed=0, route=cfg.route_classes[0], sample_y=48)
 
 
-@pytest.mark.parametrize("kernels", ["pipelined", "simple"])
+@pytest.mark.parametrize("kernels", ["fused", "pipelined", "simple"])
 @pytest.mark.parametrize("qtype", [synth.Q8_0, synth.Q4_0])
 def test_ragged_shapes_decode(qtype, kernels, monkeypatch):
-    """Rows of 6 / 10 (Q8_0) and 3 / 5 (Q4_0) 16-byte vectors: partially filled warps.  Both the
-    pipelined batch-1 kernels and the one-warp-per-row kernels (used for shapes the pipelined ones
-    do not take) are checked."""
+    """Rows of 6 / 10 (Q8_0) and 3 / 5 (Q4_0) 16-byte vectors: partially filled warps.  The fused
+    one-launch batch-1 kernel, the two pipelined kernels it replaces, and the one-warp-per-row
+    kernels (used for shapes the pipelined ones do not take) are checked."""
     if kernels == "simple":
         monkeypatch.setenv("MF_DECODE_SIMPLE", "1")
+    if kernels == "pipelined":
+        monkeypatch.setenv("MF_DECODE_UNFUSED", "1")
     shape = Shape(2, 96, 12, 3, 160, qtype, model_seed=5)
     _decode_run(shape, 4, 40, seed=3)
 
 
-def test_q4_0_decode_full_width():
+@pytest.mark.parametrize("kernels", ["fused", "pipelined"])
+def test_q4_0_decode_full_width(kernels, monkeypatch):
     """Q4_0 at hidden 2048 / intermediate 768 (the 48-layer Q4_0 shape), one layer, batch 1."""
+    if kernels == "pipelined":
+        monkeypatch.setenv("MF_DECODE_UNFUSED", "1")
     shape = Shape(1, 2048, 128, 8, 768, synth.Q4_0, model_seed=0)
     _decode_run(shape, 19, 24, seed=2, route=synth.configs.ZIPF12, sample_y=12)
 
