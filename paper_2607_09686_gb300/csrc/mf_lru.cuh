@@ -15,14 +15,16 @@ namespace mf {
 
 // State of the layer in shared memory: s_slot_of[E], s_expert_of[S_active], s_last[S_active].
 // Writes the call's access record (uniq, uslot, umiss, trace), per-wave miss lists and counts,
-// the counters and the clock.  All 32 lanes must call it; lane 0 does the writes.
+// the counters and the clock.  All 32 lanes must call it.  The accesses are decided one after
+// the other (lane 0 updates the state; the warp searches free and least-recently-used slots);
+// the record of every access is then written by the whole warp at once.
 __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const int* s_uniq, int* s_slot_of,
                                          int* s_expert_of, uint64_t* s_last, int* s_uslot, uint64_t clock) {
   const int lane = threadIdx.x & 31, E = d.E, S = d.S_active;  // the clock is kept by lane 0
-  uint64_t hits = 0, misses = 0, evictions = 0;
-  int wave_miss = 0;
+  constexpr int kMissBit = 1 << 30;                             // in s_uslot until the record is written
+  uint64_t evictions = 0;
+  int wave = 0, wpos = 0, wave_miss = 0;  // wave of access u, u's position in it, misses so far in it
   for (int u = 0; u < U; ++u) {
-    if (u % S == 0) wave_miss = 0;
     const int e = s_uniq[u];
     int s = s_slot_of[e];
     const bool hit = s >= 0;
@@ -58,34 +60,52 @@ __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const i
       if (lane == 0) {
         s_expert_of[s] = e;
         s_slot_of[e] = s;
-        d.miss_list[(u / S) * S + wave_miss] = u;
+        d.miss_list[wave * S + wave_miss] = u;
       }
       ++wave_miss;
-      ++misses;
-    } else {
-      ++hits;
     }
     if (lane == 0) {
-      if (u % S == S - 1 || u == U - 1) d.info[2 + u / S] = wave_miss;
       s_last[s] = ++clock;
-      s_uslot[u] = s;
-      d.uniq[u] = e;
-      d.uslot[u] = s;
-      d.umiss[u] = hit ? 0 : 1;
-      d.tr_expert[(size_t)layer * E + u] = e;
-      d.tr_slot[(size_t)layer * E + u] = s;
-      d.tr_hit[(size_t)layer * E + u] = hit ? 1 : 0;
+      s_uslot[u] = hit ? s : (s | kMissBit);
+    }
+    if (++wpos == S || u == U - 1) {  // end of a wave: its miss count
+      if (lane == 0) d.info[2 + wave] = wave_miss;
+      ++wave;
+      wpos = 0;
+      wave_miss = 0;
     }
     __syncwarp();  // lane 0's shared-memory updates are seen by the whole warp at the next access
   }
+  // the record of every access, and the counters
+  unsigned misses = 0;
+  for (int u0 = 0; u0 < U; u0 += 32) {  // warp-uniform: every lane takes part in the ballot
+    const int u = u0 + lane;
+    const bool valid = u < U;
+    int s = valid ? s_uslot[u] : 0;
+    const bool miss = valid && (s & kMissBit);
+    s &= ~kMissBit;
+    misses += __popc(__ballot_sync(0xffffffffu, miss));
+    if (valid) {
+      const int e = s_uniq[u];
+      s_uslot[u] = s;
+      d.uniq[u] = e;
+      d.uslot[u] = s;
+      d.umiss[u] = miss ? 1 : 0;
+      d.tr_expert[(size_t)layer * E + u] = e;
+      d.tr_slot[(size_t)layer * E + u] = s;
+      d.tr_hit[(size_t)layer * E + u] = miss ? 0 : 1;
+    }
+  }
+  __syncwarp();
   if (lane == 0) {
+    const uint64_t hits = (uint64_t)U - misses;
     d.clock[layer] = clock;
     unsigned long long* st = reinterpret_cast<unsigned long long*>(d.stats + (size_t)layer * 5);
     atomicAdd(st + 0, (unsigned long long)U);  // no return value used: fire-and-forget reductions
     atomicAdd(st + 1, (unsigned long long)hits);
     atomicAdd(st + 2, (unsigned long long)misses);
     atomicAdd(st + 3, (unsigned long long)evictions);
-    atomicAdd(st + 4, (unsigned long long)(misses * d.lay.canonical));
+    atomicAdd(st + 4, (unsigned long long)((uint64_t)misses * d.lay.canonical));
     d.info[0] = U;
     d.info[1] = (U + S - 1) / S;
     d.tr_n[layer] = U;

@@ -9,7 +9,10 @@
 // not depend on the summation order.
 //
 // One thread-block cluster of 8 blocks per token: block r computes the logits of experts
-// [r*ceil(E/8), (r+1)*ceil(E/8)) into its shared memory (one warp per expert at a time).  After
+// [r*ceil(E/8), (r+1)*ceil(E/8)) into its shared memory, with 16 / ceil(E/8) warps per expert
+// when the block has fewer experts than warps (each warp a lane-interleaved share of the row,
+// its loads issued together; the warps' compensated pairs are then added with the same
+// error-free steps).  After
 // a cluster barrier, block 0 gathers all logits through distributed shared memory, ranks each
 // expert by counting the experts ahead of it, and keeps the k first.  With one token per call,
 // block 0 then runs the layer's slot resolve (lru_warp) on cache state it prefetched into
@@ -24,7 +27,9 @@ namespace mf {
 namespace {
 
 constexpr int kClusterCtas = 8;
-constexpr int kThreadsR = 256;
+constexpr int kThreadsR = 512;
+constexpr int kWarpsR = kThreadsR / 32;
+constexpr int kChunk = 8;  // float4 loads of W (and of x) a lane issues before using them
 constexpr int kPre = kMaxExperts / kThreadsR;  // prefetched cache-state entries per thread
 
 struct F2 {
@@ -47,22 +52,34 @@ __device__ __forceinline__ void dot2(float& s, float& c, float a, float b) {
   c = __fadd_rn(c, __fadd_rn(t.lo, pe));
 }
 
-// compensated dot product of one expert row with x, whole warp; result rounded to fp32
-__device__ __forceinline__ float logit(const float* __restrict__ w, const float* __restrict__ x, int H, int lane) {
-  float s = 0.f, c = 0.f;
-  for (int i0 = lane * 4; i0 < H; i0 += 128 * 4) {
-    float4 a[4], b[4];
+// (s, c) += (s2, c2) for compensated pairs
+__device__ __forceinline__ void pair_add(float& s, float& c, float s2, float c2) {
+  const F2 t = two_sum(s, s2);
+  s = t.hi;
+  c = __fadd_rn(__fadd_rn(c, c2), t.lo);
+}
+
+// Compensated partial dot product of one expert row with x over the float4 indices
+// q = first, first + step, ... (< H / 4), summed over the warp; returns the pair in (s, c).
+__device__ __forceinline__ void logit_part(const float* __restrict__ w, const float* __restrict__ x, int n4, int first,
+                                           int step, float& s, float& c) {
+  s = 0.f;
+  c = 0.f;
+  const float4* w4 = reinterpret_cast<const float4*>(w);
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  for (int q0 = first; q0 < n4; q0 += kChunk * step) {
+    float4 a[kChunk], b[kChunk];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {  // all loads of the chunk first
-      const int i = i0 + u * 128;
-      if (i < H) {
-        a[u] = __ldg(reinterpret_cast<const float4*>(w + i));
-        b[u] = __ldg(reinterpret_cast<const float4*>(x + i));
+    for (int u = 0; u < kChunk; ++u) {  // all loads of the chunk first
+      const int q = q0 + u * step;
+      if (q < n4) {
+        a[u] = __ldg(w4 + q);
+        b[u] = __ldg(x4 + q);
       }
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (i0 + u * 128 < H) {
+    for (int u = 0; u < kChunk; ++u) {
+      if (q0 + u * step < n4) {
         dot2(s, c, a[u].x, b[u].x);
         dot2(s, c, a[u].y, b[u].y);
         dot2(s, c, a[u].z, b[u].z);
@@ -74,11 +91,8 @@ __device__ __forceinline__ float logit(const float* __restrict__ w, const float*
   for (int off = 16; off > 0; off >>= 1) {
     const float so = __shfl_xor_sync(0xffffffffu, s, off);
     const float co = __shfl_xor_sync(0xffffffffu, c, off);
-    const F2 t2 = two_sum(s, so);
-    s = t2.hi;
-    c = __fadd_rn(__fadd_rn(c, co), t2.lo);
+    pair_add(s, c, so, co);
   }
-  return __fadd_rn(s, c);
 }
 
 __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR)
@@ -93,6 +107,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
   const float* xt = x + (size_t)t * H;
 
   __shared__ float s_z[kMaxExperts];  // own logits; block 0: all logits
+  __shared__ float s_ps[kWarpsR], s_pc[kWarpsR];  // each warp's compensated partial
   __shared__ int s_sel[kMaxTopK];
   __shared__ float s_zsel[kMaxTopK];
   __shared__ int s_slot_of[kMaxExperts];
@@ -119,12 +134,26 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
   }
 
   const int e0 = rank * epc, e1 = min(E, e0 + epc);
-  for (int e = e0 + warp; e < e1; e += kThreadsR / 32) {
-    float z = logit(wr + (size_t)e * H, xt, H, lane);
+  const int wpe = epc >= kWarpsR ? 1 : kWarpsR / epc;  // warps per expert
+  const int ew = kWarpsR / wpe;                         // experts per pass
+  const int part = warp % wpe, n4 = H / 4;
+  for (int eb = e0; eb < e1; eb += ew) {  // block-uniform passes
+    const int e = eb + warp / wpe;
+    float ps = 0.f, pc = 0.f;
+    if (e < e1 && warp / wpe < ew) logit_part(wr + (size_t)e * H, xt, n4, part * 32 + lane, wpe * 32, ps, pc);
     if (lane == 0) {
+      s_ps[warp] = ps;
+      s_pc[warp] = pc;
+    }
+    __syncthreads();
+    if (lane == 0 && part == 0 && e < e1 && warp / wpe < ew) {
+      float zs = s_ps[warp], zc = s_pc[warp];
+      for (int p = 1; p < wpe; ++p) pair_add(zs, zc, s_ps[warp + p], s_pc[warp + p]);
+      float z = __fadd_rn(zs, zc);
       if (bias) z = __fadd_rn(z, bias[(size_t)t * E + e]);
       s_z[e - e0] = z;
     }
+    __syncthreads();
   }
   cluster.sync();
   if (rank == 0) {  // gather every block's logits
