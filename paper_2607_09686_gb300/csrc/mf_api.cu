@@ -506,6 +506,15 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   const bool gemm = T > 1 && c->prefill_min_t > 0 && T >= c->prefill_min_t;
   if (gemm) MF_CUDA(launch_tile_x(d, x, T, s));
 
+  if (T == 1 && c->ffn_fused) {  // one launch: expert FFN, with the misses materialised inside
+    timer_mark(c, kTFfn, 0, s);
+    MF_CUDA(launch_ffn_single(d, layer, x, y, s));
+    timer_mark(c, kTFfn, 1, s);
+    if (idx_out) MF_CUDA(cudaMemcpyAsync(idx_out, d.idx, sizeof(int32_t) * d.k, cudaMemcpyDeviceToDevice, s));
+    if (w_out) MF_CUDA(cudaMemcpyAsync(w_out, d.g, sizeof(float) * d.k, cudaMemcpyDeviceToDevice, s));
+    return MF_OK;
+  }
+
   long long accesses_max = (long long)T * d.k;
   if (accesses_max > d.E) accesses_max = d.E;
   const int n_waves = (int)((accesses_max + S - 1) / S);
@@ -529,12 +538,6 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
         MF_CUDA(launch_combine(d, T, y, s));
         timer_mark(c, kTDown, 1, s);
       }
-      continue;
-    }
-    if (T == 1 && c->ffn_fused) {
-      timer_mark(c, kTFfn, 0, s);
-      MF_CUDA(launch_ffn_single(d, layer, x, y, s));
-      timer_mark(c, kTFfn, 1, s);
       continue;
     }
     const bool pipe = T == 1 && c->decode_pipe;

@@ -35,6 +35,7 @@ constexpr int kThreads = (kConsumers + 1) * 32;
 constexpr int kMaxStages = 12;
 constexpr size_t kSmemBudget = 200 * 1024;
 constexpr size_t kFusedSmem = 224 * 1024;  // the fused kernel's dynamic + static shared memory
+constexpr int kMaxItemsF = 64;            // gate/up items one block of the fused kernel may take
 
 struct PipeCfg {
   int R;                 // rows per item
@@ -305,7 +306,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 }
 
 // ---------------------------------------------------------------- fused gate/up + down, one token
-// Both projections in one persistent cooperative launch.  A block's down work is a contiguous
+// Both projections in one persistent cooperative launch, which also materialises the call's
+// missed experts: their items are read straight from the pinned pack (the whole producer warp,
+// 16-byte loads over the host link) into the stage and written through to the expert's new HBM
+// slot, after the resident experts' items, so the resident data and the compute overlap the
+// link transfer.  A block's down work is a contiguous
 // range of rpc output rows: its item j is expert j's rpc down records, one bulk copy into a buffer
 // of its own.  The producer requests those k copies right after the first gate/up items (the down
 // weights do not depend on h), then streams the rest of the gate/up items through the ring, so the
@@ -313,6 +318,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 // their gate/up items, publish it, meet every other block at a grid-wide arrival counter (bounded
 // wait), and then take the down items with the k experts' h.  The counter never resets: each launch adds one
 // arrival per block, and a block waits for the multiple of gridDim.x that completes its launch.
+// One item of a missed expert, by the whole warp: `bytes` (a multiple of 16) from the pinned pack
+// into the shared-memory stage, every piece in flight at once (cp.async); then lane 0 writes the
+// stage through to the expert's HBM slot with one bulk copy (completion awaited before the stage
+// is refilled and before the block exits).
+__device__ __forceinline__ void host_fill(unsigned char* stage, uint8_t* slot, const uint8_t* pack, uint32_t bytes,
+                                          int lane) {
+  const int n = (int)(bytes / 16);
+  for (int i = lane; i < n; i += 32)
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(stage + (size_t)i * 16)),
+                 "l"(pack + (size_t)i * 16)
+                 : "memory");
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // before the bulk copy reads them
+  __syncwarp();
+  if (lane == 0) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(slot), "r"(smem_u32(stage)),
+                 "r"(bytes)
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+  }
+}
+// lane 0: the stage-to-slot copies issued so far have read their source (the stage may be refilled)
+__device__ __forceinline__ void slot_writes_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// ... and have completed
+__device__ __forceinline__ void slot_writes_done() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 struct FusedCfg {
   PipeCfg g;
   int rpc;               // down: output rows per block (a contiguous range)
@@ -346,9 +377,12 @@ template <int QT, int VPL, int VPLD>
 __global__ void __launch_bounds__(kThreads, 1)
     k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, float* __restrict__ y, FusedCfg f) {
   extern __shared__ __align__(128) unsigned char smem[];
-  __shared__ const uint8_t* s_gu[kMaxTopK];
-  __shared__ const uint8_t* s_dn[kMaxTopK];
+  __shared__ uint8_t* s_gu[kMaxTopK];  // each expert's HBM slot: gate/up region, down region
+  __shared__ uint8_t* s_dn[kMaxTopK];
+  __shared__ const uint8_t* s_hgu[kMaxTopK];  // its payload in the pinned pack (missed experts)
   __shared__ float s_g[kMaxTopK];
+  __shared__ int s_miss[kMaxTopK];
+  __shared__ int s_gord[kMaxItemsF];  // the block's gate/up items: resident experts' first
   const PipeCfg& cg = f.g;
   Smem sm;
   sm.stage0 = smem;
@@ -363,13 +397,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int mine_g = items_of_block(cg.n_items);
   const int r0 = (int)blockIdx.x * f.rpc, nrows = max(0, min(d.H - r0, f.rpc));  // this block's down rows
   const int mine_d = nrows > 0 ? k : 0;
-  if (threadIdx.x < k) {
-    const uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
+  if (threadIdx.x < k) {  // one token: access u = rank j
+    uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
     s_gu[threadIdx.x] = slot;
     s_dn[threadIdx.x] = slot + d.lay.d_off;
+    s_hgu[threadIdx.x] = d.pack + ((size_t)layer * d.E + d.uniq[threadIdx.x]) * d.lay.stride;
     s_g[threadIdx.x] = d.g[threadIdx.x];
+    s_miss[threadIdx.x] = d.umiss[threadIdx.x];
   }
+  __syncthreads();
   if (threadIdx.x == 0) {
+    const int nrb = d.I / cg.R;
+    int n = 0;
+    for (int pass = 0; pass < 2; ++pass)  // resident experts' items, then missed experts'
+      for (int t = 0; t < mine_g; ++t) {
+        const int item = (int)blockIdx.x + t * (int)gridDim.x;
+        if (s_miss[item / nrb] == pass) s_gord[n++] = item;
+      }
     for (int s = 0; s < f.NS; ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], kConsumers);
@@ -380,48 +424,62 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
 
   if (warp == kConsumers) {
-    if (lane == 0) {
-      const int grid = (int)gridDim.x;
-      Ring ring;
-      int it = 0;
-      bool ok = true;
-      // gate/up items: R contiguous row records of expert u; after the first ring's worth (or
-      // two items, whichever is fewer), the k down copies
-      const int R = cg.R, nrb = d.I / R;
-      const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
-      const int first = min(mine_g, min(2, f.NS));
-      int u = (int)blockIdx.x / nrb, rb = (int)blockIdx.x % nrb;
-      bool d_issued = false;
-      for (int i = 0; i < mine_g && ok; ++i, ++it) {
-        if (i == first) {
-          d_issued = true;
-          const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
-          const size_t off = (size_t)r0 * d.lay.rs_d;
-          for (int j = 0; j < mine_d; ++j) {
+    // ---- producer warp: lane 0 issues the bulk copies; all lanes fill missed experts' items
+    Ring ring;
+    int it = 0;
+    bool ok = true;
+    const int R = cg.R, nrb = d.I / R;
+    const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
+    const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
+    const size_t doff = (size_t)r0 * d.lay.rs_d;
+    // the resident experts' down records go after the first two gate/up items
+    const int first = min(mine_g, min(2, f.NS));
+    bool d_issued = false;
+    auto issue_down_hits = [&]() {
+      if (lane == 0)
+        for (int j = 0; j < mine_d; ++j)
+          if (!s_miss[j]) {
             mbar_arrive_tx(&full_d[j], dbytes);
-            bulk_g2s(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + off, dbytes, &full_d[j]);
+            bulk_g2s(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, dbytes, &full_d[j]);
           }
+      d_issued = true;
+    };
+    for (int t = 0; t < mine_g; ++t, ++it) {
+      if (t == first) issue_down_hits();
+      if (it >= f.NS) {
+        int w = 1;
+        if (lane == 0) {
+          w = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u);
+          slot_writes_read();
         }
-        if (it >= f.NS && !(ok = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u))) break;
-        uint64_t* bar = &sm.full[ring.s];
-        mbar_arrive_tx(bar, bytes);
-        bulk_g2s(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar);
-        ring.next(f.NS);
-        rb += grid;
-        while (rb >= nrb) {
-          rb -= nrb;
-          ++u;
+        if (!__shfl_sync(0xffffffffu, w, 0)) {
+          ok = false;
+          break;
         }
       }
-      if (!d_issued && ok) {  // fewer gate/up items than `first`: the down copies go now
-        const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
-        const size_t off = (size_t)r0 * d.lay.rs_d;
-        for (int j = 0; j < mine_d; ++j) {
-          mbar_arrive_tx(&full_d[j], dbytes);
-          bulk_g2s(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + off, dbytes, &full_d[j]);
+      const int item = s_gord[t], u = item / nrb, rb = item % nrb;
+      unsigned char* st = sm.stage0 + (size_t)ring.s * f.stage_bytes;
+      const size_t off = (size_t)rb * R * rs;
+      uint64_t* bar = &sm.full[ring.s];
+      if (!s_miss[u]) {
+        if (lane == 0) {
+          mbar_arrive_tx(bar, bytes);
+          bulk_g2s(st, s_gu[u] + off, bytes, bar);
         }
-        d_issued = true;
+      } else {
+        host_fill(st, s_gu[u] + off, s_hgu[u] + off, bytes, lane);  // ends with a warp barrier
+        if (lane == 0) mbar_arrive(bar);  // release: every lane's stage writes
       }
+      ring.next(f.NS);
+    }
+    if (ok && !d_issued) issue_down_hits();
+    if (ok)  // missed experts' down records
+      for (int j = 0; j < mine_d; ++j)
+        if (s_miss[j]) {
+          host_fill(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, s_hgu[j] + d.lay.d_off + doff, dbytes, lane);
+          if (lane == 0) mbar_arrive(&full_d[j]);
+        }
+    if (lane == 0) {
       if (!ok) atomicExch(d.err, 1u);
       // no copy may be in flight when the block exits: wait for the last use of every stage
       for (int s = 0; s < f.NS && s < it; ++s) {
@@ -430,7 +488,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (d_issued)
         for (int j = 0; j < mine_d; ++j)
-          if (!mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
+          if (!s_miss[j] && !mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
+      slot_writes_done();
     }
   } else {
     Ring ring;
@@ -478,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           ag += p[(0 * R + r) * cs + cc];
           au += p[(1 * R + r) * cs + cc];
         }
-        const int item = (int)blockIdx.x + it * (int)gridDim.x;
+        const int item = s_gord[it];
         d.h[(size_t)(item / nrb) * d.I + (item % nrb) * R + r] = ag / (1.0f + expf(-ag)) * au;
       }
       named_bar_sync(1, kConsumers * 32);  // the block's h written
@@ -734,7 +793,10 @@ cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStrea
 
 size_t decode_smem_bytes(const Dev& d, int which) { return smem_bytes(which == 0 ? gateup_cfg(d) : down_cfg(d)); }
 
-bool ffn_fused_ok(const Dev& d) { return decode_pipe_ok(d) && fused_cfg(d).NS >= 2; }
+bool ffn_fused_ok(const Dev& d) {
+  const FusedCfg f = fused_cfg(d);
+  return decode_pipe_ok(d) && f.NS >= 2 && f.g.max_mine <= kMaxItemsF;
+}
 
 cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
   return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, y, s) : ffn_pipe_q<kQ4>(d, layer, x, y, s);
