@@ -35,7 +35,7 @@ N_TOKENS = 256
 # DRAM bytes (read + write) of one launch of the roofline kernel (the fused one-token FFN) from
 # the ncu capture summarised under profiles/, valid while the kernel sources hash to `sha`
 # (otherwise the line reports null: the counters no longer describe the kernel that ran).
-KERNEL_TRAFFIC = {"sha": None, "bytes": None,
+KERNEL_TRAFFIC = {"sha": "3e610f36a78815b0", "bytes": 40194816,
                   "files": ("paper_2607_09686_gb300/csrc/mf_decode.cu", "paper_2607_09686_gb300/csrc/mf_dequant.cuh",
                             "paper_2607_09686_gb300/csrc/mf_internal.cuh")}
 
@@ -299,12 +299,20 @@ def run_mawforge(args):
         "roofline": {"bound": "hbm", "kernel": rf_kernel,
                      "achieved": round(rf_gbs, 1), "peak": hbm, "unit": "GB/s",
                      "frac": round(rf_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": _captured_traffic(),
-                     "bytes_per_launch": rf_bytes, "frac_of_8tbs": round(gemv_gbs / 8000.0, 4),
-                     "timing": "CUDA events around each launch in instrumented replays of the step graph"},
+                     "bytes_per_launch": rf_bytes,
+                     "bytes_note": "every launch reads its resident experts' blocks from HBM and writes its missed "
+                                   "experts' blocks to HBM: k payloads per launch; traffic is an all-resident "
+                                   "launch's ncu DRAM bytes",
+                     "timing": "CUDA events around each launch in instrumented replays of the step graph; "
+                               "launches with misses wait on the host link"},
         "kernels": kernels,
         "copy": {"materialized_bytes_per_step": st["bytes_materialized"],
                  "materialize_gbs": round(args.steps * st["bytes_materialized"] / (ms_mat * 1e-3) / 1e9, 1)
-                 if ms_mat else None},
+                 if ms_mat else None,
+                 "link_gbs_lower_bound": round(args.steps * st["bytes_materialized"] / (gemv_ms * 1e-3) / 1e9, 1)
+                 if n_ff else None,
+                 "note": "one-token calls materialise inside the fused FFN launch; the lower bound divides "
+                         "the materialised bytes by all of that kernel's time"},
         "clocks": clocks,
         "e2e": {"value": round(N_TOKENS / (statistics.mean(e2e_ms) * 1e-3) * ws, 2), "unit": "tokens/s",
                 "h2d_bytes_per_step": N_TOKENS * L * (H + E) * 4, "d2h_bytes_per_step": N_TOKENS * L * H * 4},
@@ -315,6 +323,9 @@ def run_mawforge(args):
     # the same calls), one router per call and one reset per step
     line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps * (N_TOKENS * L + 1)
     mf.mf_destroy(ctx)
+    if n_ff and not args.no_resident:
+        line["roofline"]["resident"] = resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush,
+                                                            args.steps, rf_bytes, hbm)
     if not args.no_prefill:
         line["prefill"] = prefill_measurement(torch, mf, synth, device)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -323,6 +334,57 @@ def run_mawforge(args):
         print(json.dumps(line))
     if ws > 1:
         torch.distributed.destroy_process_group()
+
+
+def resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, steps, bytes_per_launch, hbm):
+    """The same 1024 calls with every expert resident (a 100 % cache, warmed by one pass): the
+    fused FFN launch is then HBM-bound; CUDA events around each launch in graph replays."""
+    cfg = synth.CONFIGS[WORKLOAD]
+    L, H, E, k, I, q = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    model = mf.Model(L, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(100.0, 1 << 62, 0, 0, 1, 0))
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    try:
+        buf = np.empty(plan.payload_bytes, np.uint8)
+        for l in range(L):
+            for e in range(E):
+                synth.payload(cfg.model_seed, l, e, H, I, q, out=buf)
+                mf.mf_pack_put(ctx, l, e, buf)
+        y = torch.empty(N_TOKENS, L, H, device=device)
+
+        def calls():
+            for t in range(N_TOKENS):
+                for l in range(L):
+                    mf.mf_moe_forward(ctx, l, x[t, l], wr[l], bias[t, l], 1, y[t, l], None, None, stream)
+
+        with torch.cuda.stream(stream):
+            for _ in range(2):  # every expert the sequence uses becomes resident
+                calls()
+            stream.synchronize()
+            mf.mf_timing(ctx, ["ffn_fused"])
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                calls()
+        torch.cuda.synchronize()
+        mf.mf_stats(ctx, -1, reset=True)
+        ms, n = 0.0, 0
+        for i in range(3 + steps):
+            with torch.cuda.stream(stream):
+                flush.zero_()
+                g.replay()
+            r = mf.mf_timing_read(ctx)["ffn_fused"]
+            if i >= 3:
+                ms += r[0]
+                n += r[1]
+        mf.mf_timing(ctx, [])
+        st = mf.mf_stats(ctx, -1)
+    finally:
+        mf.mf_destroy(ctx)
+    us = 1e3 * ms / n
+    gbs = bytes_per_launch / (us * 1e-6) / 1e9
+    return {"achieved": round(gbs, 1), "frac": round(gbs / hbm, 4), "us_per_launch": round(us, 3), "launches": n,
+            "misses_in_timed_replays": st["misses"],
+            "how": "same calls, 100 % cache warmed by two passes (every launch all-resident), L2 flushed per replay"}
 
 
 def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: float = 15.0) -> dict:
@@ -451,6 +513,7 @@ def main():
     ap.add_argument("--cpu-tokens", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prefill", action="store_true", help="skip the 4096-token prefill measurement")
+    ap.add_argument("--no-resident", action="store_true", help="skip the all-resident FFN measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle
