@@ -148,11 +148,11 @@ int mf_moe_forward(mf_ctx_t* ctx, int layer, const float* x, const float* router
  * Host only; applies to calls issued afterwards. */
 int mf_prefill_threshold(mf_ctx_t* ctx, int min_tokens);
 
-/* As mf_moe_forward, with x, logit_bias, y, idx_out and w_out in HOST memory (pinned
- * memory lets the copies overlap; pageable memory works but serialises).  Stages x and
- * the bias into the context's device buffers, runs the step and copies the outputs back,
- * all on `stream`.  The host buffers must stay valid until the stream reaches the end of
- * the call (synchronise before reading y). */
+/* As mf_moe_forward, with x, logit_bias, y, idx_out and w_out in HOST memory.  Pageable
+ * buffers: x and the bias are staged into the context's device buffers and the outputs copied
+ * back, all on `stream`.  Pinned buffers (cudaHostAlloc / cudaHostRegister) with T = 1: no copy
+ * steps -- the kernels read x and the bias and write y over the CPU-GPU link.  The host buffers
+ * must stay valid until the stream reaches the end of the call (synchronise before reading y). */
 int mf_moe_forward_host(mf_ctx_t* ctx, int layer, const float* x, const float* router_w,
                         const float* logit_bias, int T, float* y, int32_t* idx_out, float* w_out,
                         void* stream);

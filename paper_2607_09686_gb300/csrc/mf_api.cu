@@ -585,6 +585,29 @@ int mf_moe_forward_host(mf_ctx_t* c, int layer, const float* x, const float* rou
   if (!guard.ok) return cuda_fail(cudaSetDevice(c->device), "cudaSetDevice");
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   const Dev& d = c->d;
+  // One token with pinned buffers: no copy steps.  The router reads x and the bias over the
+  // CPU-GPU link (x once per block) and leaves a device copy of x for the FFN, which writes y
+  // straight into the caller's buffer.
+  if (T == 1 && c->ffn_fused && !(((uintptr_t)x | (uintptr_t)router_w) & 15)) {
+    void *xd = nullptr, *bd = nullptr, *yd = nullptr;
+    bool pinned = cudaHostGetDevicePointer(&xd, const_cast<float*>(x), 0) == cudaSuccess &&
+                  cudaHostGetDevicePointer(&yd, y, 0) == cudaSuccess &&
+                  (!logit_bias || cudaHostGetDevicePointer(&bd, const_cast<float*>(logit_bias), 0) == cudaSuccess);
+    if (!pinned) cudaGetLastError();  // pageable memory: not an error, the copy path below serves it
+    if (pinned && !(reinterpret_cast<uintptr_t>(xd) & 15)) {
+      if (__atomic_load_n(&c->n_put, __ATOMIC_ACQUIRE) != (int64_t)d.L * d.E) return MF_E_STATE;
+      timer_mark(c, kTRouter, 0, s);
+      MF_CUDA(launch_router(d, static_cast<const float*>(xd), router_w, static_cast<const float*>(bd), 1, layer, s,
+                            c->stage_x));
+      timer_mark(c, kTRouter, 1, s);
+      timer_mark(c, kTFfn, 0, s);
+      MF_CUDA(launch_ffn_single(d, layer, c->stage_x, static_cast<float*>(yd), s));
+      timer_mark(c, kTFfn, 1, s);
+      if (idx_out) MF_CUDA(cudaMemcpyAsync(idx_out, d.idx, sizeof(int32_t) * d.k, cudaMemcpyDeviceToHost, s));
+      if (w_out) MF_CUDA(cudaMemcpyAsync(w_out, d.g, sizeof(float) * d.k, cudaMemcpyDeviceToHost, s));
+      return MF_OK;
+    }
+  }
   MF_CUDA(cudaMemcpyAsync(c->stage_x, x, sizeof(float) * T * d.H, cudaMemcpyHostToDevice, s));
   if (logit_bias)
     MF_CUDA(cudaMemcpyAsync(c->stage_bias, logit_bias, sizeof(float) * T * d.E, cudaMemcpyHostToDevice, s));

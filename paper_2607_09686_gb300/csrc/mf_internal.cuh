@@ -168,8 +168,9 @@ Layout make_layout(const mf_model_t& m);
 uint64_t canonical_payload_bytes(const mf_model_t& m);
 
 // kernel launchers (each returns the launch status)
+// x and bias may be pinned host memory; with x_copy, the router also writes x there (device)
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
-                          cudaStream_t s);
+                          cudaStream_t s, float* x_copy = nullptr);
 cudaError_t launch_resolve(const Dev& d, int layer, int T, cudaStream_t s);
 cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s);
 cudaError_t launch_gateup(const Dev& d, int layer, int wave, int wave_width, const float* x, cudaStream_t s);

@@ -59,14 +59,14 @@ __device__ __forceinline__ void pair_add(float& s, float& c, float s2, float c2)
   c = __fadd_rn(__fadd_rn(c, c2), t.lo);
 }
 
-// Compensated partial dot product of one expert row with x over the float4 indices
-// q = first, first + step, ... (< H / 4), summed over the warp; returns the pair in (s, c).
-__device__ __forceinline__ void logit_part(const float* __restrict__ w, const float* __restrict__ x, int n4, int first,
-                                           int step, float& s, float& c) {
+// Compensated partial dot product of one expert row with x (in shared memory) over the float4
+// indices q = first, first + step, ... (< H / 4), summed over the warp; returns the pair in (s, c).
+__device__ __forceinline__ void logit_part(const float* __restrict__ w, const float* xs, int n4, int first, int step,
+                                           float& s, float& c) {
   s = 0.f;
   c = 0.f;
   const float4* w4 = reinterpret_cast<const float4*>(w);
-  const float4* x4 = reinterpret_cast<const float4*>(x);
+  const float4* x4 = reinterpret_cast<const float4*>(xs);
   for (int q0 = first; q0 < n4; q0 += kChunk * step) {
     float4 a[kChunk], b[kChunk];
 #pragma unroll
@@ -74,7 +74,7 @@ __device__ __forceinline__ void logit_part(const float* __restrict__ w, const fl
       const int q = q0 + u * step;
       if (q < n4) {
         a[u] = __ldg(w4 + q);
-        b[u] = __ldg(x4 + q);
+        b[u] = x4[q];
       }
     }
 #pragma unroll
@@ -95,16 +95,32 @@ __device__ __forceinline__ void logit_part(const float* __restrict__ w, const fl
   }
 }
 
+__device__ __forceinline__ bool cluster_rank_zero() {
+  uint32_t r;
+  asm("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r == 0;
+}
+
 __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR)
     k_router(Dev d, const float* __restrict__ x, const float* __restrict__ wr, const float* __restrict__ bias, int T,
-             int layer, int fuse_resolve) {
+             int layer, int fuse_resolve, float* __restrict__ x_copy) {
+  extern __shared__ __align__(16) float s_x[];  // the token's x, read once per block
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
   const int t = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int H = d.H, E = d.E, k = d.k, S = d.S_active;
   const int epc = (E + kClusterCtas - 1) / kClusterCtas;
-  const float* xt = x + (size_t)t * H;
+  {  // x may be pinned host memory read over the CPU-GPU link: once per block
+    const float4* x4 = reinterpret_cast<const float4*>(x + (size_t)t * H);
+    float4* sx4 = reinterpret_cast<float4*>(s_x);
+    for (int i = threadIdx.x; i < H / 4; i += kThreadsR) {
+      const float4 v = x4[i];
+      sx4[i] = v;
+      if (x_copy && cluster_rank_zero()) reinterpret_cast<float4*>(x_copy + (size_t)t * H)[i] = v;  // for the FFN
+    }
+  }
+  __syncthreads();
 
   __shared__ float s_z[kMaxExperts];  // own logits; block 0: all logits
   __shared__ float s_ps[kWarpsR], s_pc[kWarpsR];  // each warp's compensated partial
@@ -140,7 +156,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
   for (int eb = e0; eb < e1; eb += ew) {  // block-uniform passes
     const int e = eb + warp / wpe;
     float ps = 0.f, pc = 0.f;
-    if (e < e1 && warp / wpe < ew) logit_part(wr + (size_t)e * H, xt, n4, part * 32 + lane, wpe * 32, ps, pc);
+    if (e < e1 && warp / wpe < ew) logit_part(wr + (size_t)e * H, s_x, n4, part * 32 + lane, wpe * 32, ps, pc);
     if (lane == 0) {
       s_ps[warp] = ps;
       s_pc[warp] = pc;
@@ -228,9 +244,12 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
 }  // namespace
 
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
-                          cudaStream_t s) {
+                          cudaStream_t s, float* x_copy) {
+  const size_t smem = (size_t)d.H * sizeof(float);
+  const cudaError_t e = cudaFuncSetAttribute(k_router, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
   dim3 grid(kClusterCtas, T);
-  k_router<<<grid, kThreadsR, 0, s>>>(d, x, wr, bias, T, layer, T == 1 ? 1 : 0);
+  k_router<<<grid, kThreadsR, smem, s>>>(d, x, wr, bias, T, layer, T == 1 ? 1 : 0, x_copy);
   return cudaGetLastError();
 }
 

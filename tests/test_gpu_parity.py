@@ -161,6 +161,45 @@ def test_host_buffer_entry_point_matches_device_entry_point():
         b.close()
 
 
+@pytest.mark.parametrize("pinned", [True, False])
+def test_host_entry_point_one_token(pinned):
+    """One token per call through the host-buffer entry point, with pinned buffers (the kernels
+    read x and the bias and write y over the CPU-GPU link, no copy steps) and with pageable ones
+    (staged copies): bit-identical to the device entry point, misses included."""
+    shape = Shape(2, 1024, 32, 8, 512, synth.Q8_0, model_seed=6)
+    a, b = Ctx(shape, 12, max_tokens=1), Ctx(shape, 12, max_tokens=1)
+    try:
+        import torch
+        import paper_2607_09686_gb300 as mf
+        T = 16
+        for l in range(shape.n_layers):
+            xs = synth.activations(2, l, 0, 0, T, shape.hidden)
+            bs = synth.plant_bias(synth.routes(2, l, 0, shape.n_experts, shape.top_k, T, 1.1, 0.3), shape.n_experts)
+            for t in range(T):
+                y1, i1, w1 = a.forward(l, xs[t:t + 1], bs[t:t + 1], 1)
+                if pinned:
+                    xh = torch.from_numpy(xs[t:t + 1].copy()).pin_memory()
+                    bh = torch.from_numpy(bs[t:t + 1].copy()).pin_memory()
+                    yh = torch.empty(1, shape.hidden).pin_memory()
+                    ih = torch.empty(1, shape.top_k, dtype=torch.int32).pin_memory()
+                    wh = torch.empty(1, shape.top_k).pin_memory()
+                    mf.mf_moe_forward_host(b.h, l, xh, b.wr[l], bh, 1, yh, ih, wh)
+                    torch.cuda.synchronize()
+                    y2, i2, w2 = yh.numpy(), ih.numpy(), wh.numpy()
+                else:
+                    y2 = np.empty_like(y1)
+                    i2 = np.empty_like(i1)
+                    w2 = np.empty_like(w1)
+                    mf.mf_moe_forward_host(b.h, l, xs[t:t + 1].copy(), b.wr[l], bs[t:t + 1].copy(), 1, y2, i2, w2)
+                    torch.cuda.synchronize()
+                assert np.array_equal(y1, y2) and np.array_equal(i1, i2) and np.array_equal(w1, w2), (l, t)
+        assert mf.mf_check(b.h) == 0
+        assert mf.mf_stats(a.h) == mf.mf_stats(b.h) and mf.mf_stats(a.h)["misses"] > 0
+    finally:
+        a.close()
+        b.close()
+
+
 def test_reset_replays_and_empty_step():
     cfg = synth.CONFIGS["tiny"]
     ctx = Ctx(Shape.of(cfg), 4, max_tokens=4)
