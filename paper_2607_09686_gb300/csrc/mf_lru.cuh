@@ -24,7 +24,28 @@ __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const i
   constexpr int kMissBit = 1 << 30;                             // in s_uslot until the record is written
   uint64_t evictions = 0;
   int wave = 0, wpos = 0, wave_miss = 0;  // wave of access u, u's position in it, misses so far in it
-  for (int u = 0; u < U; ++u) {
+  // Every access a hit (the common case): nothing is placed or evicted, so the decisions are
+  // independent -- access u just takes clock value clock + u + 1 -- and the warp applies them
+  // together.  Any miss: the accesses are walked in order (a miss may evict the slot of a later
+  // access of the same call).
+  bool all_hit = true;
+  for (int u0 = 0; u0 < U && all_hit; u0 += 32)
+    all_hit = __all_sync(0xffffffffu, u0 + lane >= U || s_slot_of[s_uniq[u0 + lane]] >= 0);
+  if (all_hit) {
+    for (int u0 = 0; u0 < U; u0 += 32) {
+      const int u = u0 + lane;
+      if (u < U) {
+        const int sl = s_slot_of[s_uniq[u]];
+        s_last[sl] = clock + (uint64_t)u + 1;
+        s_uslot[u] = sl;
+      }
+    }
+    clock += (uint64_t)U;
+    if (lane == 0)
+      for (int w = 0; w * S < U; ++w) d.info[2 + w] = 0;
+    __syncwarp();
+  }
+  for (int u = 0; u < U && !all_hit; ++u) {
     const int e = s_uniq[u];
     int s = s_slot_of[e];
     const bool hit = s >= 0;

@@ -8,11 +8,12 @@
 // where the exact value lies within ~n*2^-48 relative of a rounding boundary, so selection does
 // not depend on the summation order.
 //
-// One thread-block cluster of 8 blocks per token: block r computes the logits of experts
-// [r*ceil(E/8), (r+1)*ceil(E/8)) into its shared memory, with 16 / ceil(E/8) warps per expert
+// One thread-block cluster of 16 blocks per token (8 where the GPU does not schedule clusters of
+// 16): block r computes the logits of experts [r*ceil(E/nc), (r+1)*ceil(E/nc)), with
+// 16 / ceil(E/nc) warps per expert
 // when the block has fewer experts than warps (each warp a lane-interleaved share of the row,
 // its loads issued together; the warps' compensated pairs are then added with the same
-// error-free steps).  After
+// error-free steps), and stores them straight into block 0's shared memory.  After
 // a cluster barrier, block 0 gathers all logits through distributed shared memory, ranks each
 // expert by counting the experts ahead of it, and keeps the k first.  With one token per call,
 // block 0 then runs the layer's slot resolve (lru_warp) on cache state it prefetched into
@@ -26,7 +27,6 @@ namespace cg = cooperative_groups;
 namespace mf {
 namespace {
 
-constexpr int kClusterCtas = 8;
 constexpr int kThreadsR = 512;
 constexpr int kWarpsR = kThreadsR / 32;
 constexpr int kChunk = 8;  // float4 loads of W (and of x) a lane issues before using them
@@ -59,10 +59,21 @@ __device__ __forceinline__ void pair_add(float& s, float& c, float s2, float c2)
   c = __fadd_rn(__fadd_rn(c, c2), t.lo);
 }
 
+// The first chunk of logit_part's W loads, issued before x is in shared memory.
+__device__ __forceinline__ void w_preload(const float* __restrict__ w, int n4, int first, int step, float4* a) {
+  const float4* w4 = reinterpret_cast<const float4*>(w);
+#pragma unroll
+  for (int u = 0; u < kChunk; ++u) {
+    const int q = first + u * step;
+    if (q < n4) a[u] = __ldg(w4 + q);
+  }
+}
+
 // Compensated partial dot product of one expert row with x (in shared memory) over the float4
 // indices q = first, first + step, ... (< H / 4), summed over the warp; returns the pair in (s, c).
+// `pre` holds the first chunk's W values (w_preload).
 __device__ __forceinline__ void logit_part(const float* __restrict__ w, const float* xs, int n4, int first, int step,
-                                           float& s, float& c) {
+                                           const float4* pre, float& s, float& c) {
   s = 0.f;
   c = 0.f;
   const float4* w4 = reinterpret_cast<const float4*>(w);
@@ -73,7 +84,7 @@ __device__ __forceinline__ void logit_part(const float* __restrict__ w, const fl
     for (int u = 0; u < kChunk; ++u) {  // all loads of the chunk first
       const int q = q0 + u * step;
       if (q < n4) {
-        a[u] = __ldg(w4 + q);
+        a[u] = q0 == first ? pre[u] : __ldg(w4 + q);
         b[u] = x4[q];
       }
     }
@@ -101,16 +112,23 @@ __device__ __forceinline__ bool cluster_rank_zero() {
   return r == 0;
 }
 
-__global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR)
+__global__ void __launch_bounds__(kThreadsR)
     k_router(Dev d, const float* __restrict__ x, const float* __restrict__ wr, const float* __restrict__ bias, int T,
-             int layer, int fuse_resolve, float* __restrict__ x_copy) {
+             int layer, int fuse_resolve, float* __restrict__ x_copy, int nc) {
   extern __shared__ __align__(16) float s_x[];  // the token's x, read once per block
   cg::cluster_group cluster = cg::this_cluster();
   const int rank = (int)cluster.block_rank();
   const int t = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int H = d.H, E = d.E, k = d.k, S = d.S_active;
-  const int epc = (E + kClusterCtas - 1) / kClusterCtas;
+  const int epc = (E + nc - 1) / nc;
+  // this warp's first expert and its first W chunk, requested before x is staged
+  const int e0 = rank * epc, e1 = min(E, e0 + epc);
+  const int wpe = epc >= kWarpsR ? 1 : kWarpsR / epc;  // warps per expert
+  const int ew = kWarpsR / wpe;                         // experts per pass
+  const int part = warp % wpe, n4 = H / 4;
+  float4 pre[kChunk];
+  if (e0 + warp / wpe < e1 && warp / wpe < ew) w_preload(wr + (size_t)(e0 + warp / wpe) * H, n4, part * 32 + lane, wpe * 32, pre);
   {  // x may be pinned host memory read over the CPU-GPU link: once per block
     const float4* x4 = reinterpret_cast<const float4*>(x + (size_t)t * H);
     float4* sx4 = reinterpret_cast<float4*>(s_x);
@@ -122,7 +140,7 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
   }
   __syncthreads();
 
-  __shared__ float s_z[kMaxExperts];  // own logits; block 0: all logits
+  __shared__ __align__(16) float s_z[kMaxExperts];  // block 0: every logit (the blocks store theirs)
   __shared__ float s_ps[kWarpsR], s_pc[kWarpsR];  // each warp's compensated partial
   __shared__ int s_sel[kMaxTopK];
   __shared__ float s_zsel[kMaxTopK];
@@ -149,14 +167,14 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
     if (tid == 0) clock0 = d.clock[layer];
   }
 
-  const int e0 = rank * epc, e1 = min(E, e0 + epc);
-  const int wpe = epc >= kWarpsR ? 1 : kWarpsR / epc;  // warps per expert
-  const int ew = kWarpsR / wpe;                         // experts per pass
-  const int part = warp % wpe, n4 = H / 4;
+  float* z0 = rank == 0 ? s_z : cluster.map_shared_rank(s_z, 0);  // block 0's logits
   for (int eb = e0; eb < e1; eb += ew) {  // block-uniform passes
     const int e = eb + warp / wpe;
     float ps = 0.f, pc = 0.f;
-    if (e < e1 && warp / wpe < ew) logit_part(wr + (size_t)e * H, s_x, n4, part * 32 + lane, wpe * 32, ps, pc);
+    if (e < e1 && warp / wpe < ew) {
+      if (eb != e0) w_preload(wr + (size_t)e * H, n4, part * 32 + lane, wpe * 32, pre);
+      logit_part(wr + (size_t)e * H, s_x, n4, part * 32 + lane, wpe * 32, pre, ps, pc);
+    }
     if (lane == 0) {
       s_ps[warp] = ps;
       s_pc[warp] = pc;
@@ -167,27 +185,39 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
       for (int p = 1; p < wpe; ++p) pair_add(zs, zc, s_ps[warp + p], s_pc[warp + p]);
       float z = __fadd_rn(zs, zc);
       if (bias) z = __fadd_rn(z, bias[(size_t)t * E + e]);
-      s_z[e - e0] = z;
+      z0[e] = z;  // distributed shared memory store into block 0
     }
     __syncthreads();
   }
-  cluster.sync();
-  if (rank == 0) {  // gather every block's logits
-    for (int e = tid; e < E; e += kThreadsR) {
-      const int r = e / epc;
-      const float* src = r == 0 ? s_z : cluster.map_shared_rank(s_z, r);
-      const float z = src[e - r * epc];
-      if (r != 0) s_z[e] = z;
+  if (resolve) {  // the prefetched cache state into shared memory (the loads have long landed)
+#pragma unroll
+    for (int i = 0; i < kPre; ++i) {
+      const int e = tid + i * kThreadsR;
+      if (e < E) s_slot_of[e] = pre_slot[i];
+      if (e < S) {
+        s_expert_of[e] = pre_exp[i];
+        s_lastuse[e] = pre_last[i];
+      }
     }
   }
-  cluster.sync();  // no block leaves while block 0 may still read its shared memory
+  // every block's logits stores, before block 0 reads them; the other blocks leave
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
   if (rank != 0) return;
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 
   // rank by counting: position of expert e = experts with a larger logit, or equal and lower id
   for (int e = tid; e < E; e += kThreadsR) {
     const float z = s_z[e];
     int r = 0;
-    for (int e2 = 0; e2 < E; ++e2) {
+    for (int e4 = 0; e4 < E / 4; ++e4) {  // s_z is 16-byte aligned; E % 4 tail below
+      const float4 z4 = reinterpret_cast<const float4*>(s_z)[e4];
+      const int b = 4 * e4;
+      r += (z4.x > z) || (z4.x == z && b < e);
+      r += (z4.y > z) || (z4.y == z && b + 1 < e);
+      r += (z4.z > z) || (z4.z == z && b + 2 < e);
+      r += (z4.w > z) || (z4.w == z && b + 3 < e);
+    }
+    for (int e2 = E & ~3; e2 < E; ++e2) {
       const float z2 = s_z[e2];
       r += (z2 > z) || (z2 == z && e2 < e);
     }
@@ -197,30 +227,20 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
     }
   }
   __syncthreads();
-  if (tid == 0) {
-    float den = 0.f, ex[kMaxTopK];
-    for (int j = 0; j < k; ++j) {
-      ex[j] = expf(s_zsel[j] - s_zsel[0]);
-      den += ex[j];
-    }
-    for (int j = 0; j < k; ++j) {
-      d.idx[(size_t)t * k + j] = s_sel[j];
-      d.g[(size_t)t * k + j] = ex[j] / den;
+  if (warp == 0) {  // softmax over the chosen: lane j < k holds exp(z_j - z_0); fixed shuffle-tree sum
+    const float ex = lane < k ? expf(s_zsel[lane] - s_zsel[0]) : 0.f;
+    float den = ex;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+    if (lane < k) {
+      d.idx[(size_t)t * k + lane] = s_sel[lane];
+      d.g[(size_t)t * k + lane] = ex / den;
     }
   }
   if (!resolve) return;
 
   // One token per call: the k chosen experts are distinct, so the accesses are the chosen
   // experts in rank order, all in one wave.
-#pragma unroll
-  for (int i = 0; i < kPre; ++i) {
-    const int e = tid + i * kThreadsR;
-    if (e < E) s_slot_of[e] = pre_slot[i];
-    if (e < S) {
-      s_expert_of[e] = pre_exp[i];
-      s_lastuse[e] = pre_last[i];
-    }
-  }
   if (tid == 0) d.info[2] = 0;
   __syncthreads();
   if (warp == 0) lru_warp(d, layer, k, s_sel, s_slot_of, s_expert_of, s_lastuse, s_uslot, __shfl_sync(0xffffffffu, clock0, 0));
@@ -246,11 +266,34 @@ __global__ void __cluster_dims__(kClusterCtas, 1, 1) __launch_bounds__(kThreadsR
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
                           cudaStream_t s, float* x_copy) {
   const size_t smem = (size_t)d.H * sizeof(float);
-  const cudaError_t e = cudaFuncSetAttribute(k_router, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(k_router, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  dim3 grid(kClusterCtas, T);
-  k_router<<<grid, kThreadsR, smem, s>>>(d, x, wr, bias, T, layer, T == 1 ? 1 : 0, x_copy);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(kThreadsR);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // cluster size: 16 where the GPU can hold such a cluster (asked once), else the portable 8
+  static int nc = 0;
+  if (nc == 0) {
+    nc = 8;
+    if (cudaFuncSetAttribute(k_router, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+      cfg.gridDim = dim3(16, 1);
+      attr[0].val.clusterDim.x = 16;
+      int clusters = 0;
+      if (cudaOccupancyMaxActiveClusters(&clusters, k_router, &cfg) == cudaSuccess && clusters >= 1) nc = 16;
+    }
+    cudaGetLastError();
+  }
+  cfg.gridDim = dim3(nc, T);
+  attr[0].val.clusterDim.x = nc;
+  e = cudaLaunchKernelEx(&cfg, k_router, d, x, wr, bias, T, layer, T == 1 ? 1 : 0, x_copy, nc);
+  return e;
 }
 
 }  // namespace mf
