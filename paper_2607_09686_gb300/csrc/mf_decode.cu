@@ -32,6 +32,7 @@ using namespace dq;
 
 constexpr int kConsumers = 16;
 constexpr int kThreads = (kConsumers + 1) * 32;
+constexpr int kThreadsF = (kConsumers + 2) * 32;  // fused kernel: + a link warp
 constexpr int kMaxStages = 12;
 constexpr size_t kSmemBudget = 200 * 1024;
 constexpr size_t kFusedSmem = 224 * 1024;  // the fused kernel's dynamic + static shared memory
@@ -307,10 +308,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 
 // ---------------------------------------------------------------- fused gate/up + down, one token
 // Both projections in one persistent cooperative launch, which also materialises the call's
-// missed experts: their items are read straight from the pinned pack (the whole producer warp,
-// 16-byte loads over the host link) into the stage and written through to the expert's new HBM
-// slot, after the resident experts' items, so the resident data and the compute overlap the
-// link transfer.  A block's down work is a contiguous
+// missed experts.  The gate/up items are dealt round-robin over the blocks from a list that
+// holds the resident experts' items first, so every block gets an equal share (+-1) of the
+// missed ones.  The producer warp streams the resident items from HBM through ring A; a link
+// warp, from the first cycle, reads the missed items straight from the pinned pack (16-byte
+// loads over the host link) into the stages of a small ring B and writes each through to the
+// expert's new HBM slot, then does the same for the missed experts' down records, so the link
+// transfer overlaps the resident data and all compute.  The consumers take ring A's items, then
+// ring B's.  A block's down work is a contiguous
 // range of rpc output rows: its item j is expert j's rpc down records, one bulk copy into a buffer
 // of its own.  The producer requests those k copies right after the first gate/up items (the down
 // weights do not depend on h), then streams the rest of the gate/up items through the ring, so the
@@ -374,7 +379,7 @@ __device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, uns
 }
 
 template <int QT, int VPL, int VPLD>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreadsF, 1)
     k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, float* __restrict__ y, FusedCfg f) {
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ uint8_t* s_gu[kMaxTopK];  // each expert's HBM slot: gate/up region, down region
@@ -383,6 +388,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   __shared__ float s_g[kMaxTopK];
   __shared__ int s_miss[kMaxTopK];
   __shared__ int s_gord[kMaxItemsF];  // the block's gate/up items: resident experts' first
+  __shared__ int s_ord[kMaxTopK];     // ranks: resident experts', then missed experts'
+  __shared__ int s_nres, s_nb;        // how many of them are resident; ring B's stages
   const PipeCfg& cg = f.g;
   Smem sm;
   sm.stage0 = smem;
@@ -407,13 +414,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
   if (threadIdx.x == 0) {
+    // list position p = blockIdx.x + t * gridDim.x; the list holds the resident experts' items,
+    // then the missed experts' (ranks in order within each); item id = rank * (I / R) + row block
     const int nrb = d.I / cg.R;
-    int n = 0;
-    for (int pass = 0; pass < 2; ++pass)  // resident experts' items, then missed experts'
-      for (int t = 0; t < mine_g; ++t) {
-        const int item = (int)blockIdx.x + t * (int)gridDim.x;
-        if (s_miss[item / nrb] == pass) s_gord[n++] = item;
-      }
+    int* ord = s_ord;
+    int n_res_e = 0;
+    for (int j = 0; j < k; ++j)
+      if (!s_miss[j]) ord[n_res_e++] = j;
+    for (int j = 0, n = n_res_e; j < k; ++j)
+      if (s_miss[j]) ord[n++] = j;
+    int nres = 0;
+    for (int t = 0; t < mine_g; ++t) {
+      const int p = (int)blockIdx.x + t * (int)gridDim.x;
+      s_gord[t] = ord[p / nrb] * nrb + p % nrb;
+      nres += p < n_res_e * nrb;
+    }
+    s_nres = nres;
+    s_nb = n_res_e < k ? 2 : 0;  // ring B only when the call has a missed expert (NS >= 4)
     for (int s = 0; s < f.NS; ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], kConsumers);
@@ -423,8 +440,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   __syncthreads();
 
+  const int nres = s_nres, NB = s_nb, NA = f.NS - NB;  // ring A: stages [0, NA); ring B: [NA, NS)
   if (warp == kConsumers) {
-    // ---- producer warp: lane 0 issues the bulk copies; all lanes fill missed experts' items
+    // ---- producer warp: lane 0 streams the resident experts' items and down records
     Ring ring;
     int it = 0;
     bool ok = true;
@@ -433,7 +451,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
     const size_t doff = (size_t)r0 * d.lay.rs_d;
     // the resident experts' down records go after the first two gate/up items
-    const int first = min(mine_g, min(2, f.NS));
+    const int first = min(nres, min(2, NA));
     bool d_issued = false;
     auto issue_down_hits = [&]() {
       if (lane == 0)
@@ -444,13 +462,41 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
       d_issued = true;
     };
-    for (int t = 0; t < mine_g; ++t, ++it) {
-      if (t == first) issue_down_hits();
-      if (it >= f.NS) {
+    if (lane == 0) {
+      for (int t = 0; t < nres; ++t, ++it) {
+        if (t == first) issue_down_hits();
+        if (it >= NA && !(ok = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u))) break;
+        const int item = s_gord[t], u = item / nrb, rb = item % nrb;
+        uint64_t* bar = &sm.full[ring.s];
+        mbar_arrive_tx(bar, bytes);
+        bulk_g2s(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar);
+        ring.next(NA);
+      }
+      if (ok && !d_issued) issue_down_hits();
+      if (!ok) atomicExch(d.err, 1u);
+      // no copy may be in flight when the block exits: wait for the last use of every stage
+      for (int s = 0; s < NA && s < it; ++s) {
+        const int uses = (it - 1 - s) / NA + 1;
+        if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u)) atomicExch(d.err, 2u);
+      }
+      if (d_issued)
+        for (int j = 0; j < mine_d; ++j)
+          if (!s_miss[j] && !mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
+    }
+  } else if (warp == kConsumers + 1) {
+    // ---- link warp: the missed experts' items through ring B, then their down records
+    Ring ring;
+    bool ok = true;
+    const int R = cg.R, nrb = d.I / R;
+    const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
+    const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
+    const size_t doff = (size_t)r0 * d.lay.rs_d;
+    for (int t = nres, it = 0; t < mine_g; ++t, ++it) {
+      if (it >= NB) {
         int w = 1;
         if (lane == 0) {
-          w = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u);
-          slot_writes_read();
+          w = mbar_wait(&sm.empty[NA + ring.s], ring.phase ^ 1u);
+          slot_writes_read();  // the stage's previous write-through has read it
         }
         if (!__shfl_sync(0xffffffffu, w, 0)) {
           ok = false;
@@ -458,22 +504,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       const int item = s_gord[t], u = item / nrb, rb = item % nrb;
-      unsigned char* st = sm.stage0 + (size_t)ring.s * f.stage_bytes;
       const size_t off = (size_t)rb * R * rs;
-      uint64_t* bar = &sm.full[ring.s];
-      if (!s_miss[u]) {
-        if (lane == 0) {
-          mbar_arrive_tx(bar, bytes);
-          bulk_g2s(st, s_gu[u] + off, bytes, bar);
-        }
-      } else {
-        host_fill(st, s_gu[u] + off, s_hgu[u] + off, bytes, lane);  // ends with a warp barrier
-        if (lane == 0) mbar_arrive(bar);  // release: every lane's stage writes
-      }
-      ring.next(f.NS);
+      host_fill(sm.stage0 + (size_t)(NA + ring.s) * f.stage_bytes, s_gu[u] + off, s_hgu[u] + off, bytes,
+                lane);                                      // ends with a warp barrier
+      if (lane == 0) mbar_arrive(&sm.full[NA + ring.s]);  // release: every lane's stage writes
+      ring.next(NB);
     }
-    if (ok && !d_issued) issue_down_hits();
-    if (ok)  // missed experts' down records
+    if (ok)
       for (int j = 0; j < mine_d; ++j)
         if (s_miss[j]) {
           host_fill(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, s_hgu[j] + d.lay.d_off + doff, dbytes, lane);
@@ -481,18 +518,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     if (lane == 0) {
       if (!ok) atomicExch(d.err, 1u);
-      // no copy may be in flight when the block exits: wait for the last use of every stage
-      for (int s = 0; s < f.NS && s < it; ++s) {
-        const int uses = (it - 1 - s) / f.NS + 1;
-        if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u)) atomicExch(d.err, 2u);
-      }
-      if (d_issued)
-        for (int j = 0; j < mine_d; ++j)
-          if (!s_miss[j] && !mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
-      slot_writes_done();
+      slot_writes_done();  // every write-through complete before the block exits
     }
   } else {
-    Ring ring;
+    Ring ring, ring_b;
     bool ok = true;
     // ---- gate/up: warp w: tensor w / (R*cs), row (w / cs) % R, column range w % cs
     {
@@ -510,8 +539,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (v < nv) xr[i] = xq[v0 + v];
       }
       for (int it = 0; it < mine_g; ++it) {
-        if (!(ok = mbar_wait(&sm.full[ring.s], ring.phase))) break;
-        const unsigned char* rec = sm.stage0 + (size_t)ring.s * f.stage_bytes + row * rs;
+        const bool link = it >= nres;  // a missed expert's item: ring B
+        const int bi = link ? NA + ring_b.s : ring.s;
+        if (!(ok = mbar_wait(&sm.full[bi], link ? ring_b.phase : ring.phase))) break;
+        const unsigned char* rec = sm.stage0 + (size_t)bi * f.stage_bytes + row * rs;
         const unsigned char* q = rec + ten * d.lay.o_up + 16 * v0;
         const __half* sc = reinterpret_cast<const __half*>(rec + (ten ? d.lay.o_us : d.lay.o_gs));
         float acc = 0.f;
@@ -525,8 +556,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         acc = warp_sum(acc);
         if (lane == 0) sm.red[it * kConsumers + warp] = acc;
         __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.empty[ring.s]);
-        ring.next(f.NS);
+        if (lane == 0) mbar_arrive(&sm.empty[bi]);
+        if (link)
+          ring_b.next(NB);
+        else
+          ring.next(NA);
       }
       named_bar_sync(1, kConsumers * 32);
       for (int t = threadIdx.x; t < mine_g * R; t += kConsumers * 32) {
@@ -742,7 +776,7 @@ cudaError_t launch_coop(Kern kern, size_t smem, cudaStream_t s, const Dev& d, in
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(sm_count());
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(kThreadsF);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -795,7 +829,7 @@ size_t decode_smem_bytes(const Dev& d, int which) { return smem_bytes(which == 0
 
 bool ffn_fused_ok(const Dev& d) {
   const FusedCfg f = fused_cfg(d);
-  return decode_pipe_ok(d) && f.NS >= 2 && f.g.max_mine <= kMaxItemsF;
+  return decode_pipe_ok(d) && f.NS >= 4 && f.g.max_mine <= kMaxItemsF;
 }
 
 cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
