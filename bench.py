@@ -409,10 +409,10 @@ def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: flo
         wr = torch.from_numpy(synth.router_weights(cfg.model_seed, 0, E, H)).to(device)
         y = torch.empty(T, H, device=device)
         stream = torch.cuda.Stream(device)
-        gemm_ms, call_ms, mat_ms, n_gemm = [], [], [], 0
+        gemm_ms, call_ms, mat_ms, rt_ms, rs_ms, n_gemm = [], [], [], [], [], 0
         for i in range(calls + 1):
             mf.mf_reset(ctx, 0, stream)
-            mf.mf_timing(ctx, ["materialize", "prefill_gemm"])
+            mf.mf_timing(ctx, ["router", "resolve", "materialize", "prefill_gemm"])
             a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             with torch.cuda.stream(stream):
                 a.record(stream)
@@ -423,6 +423,8 @@ def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: flo
             if i > 0:
                 gemm_ms.append(tm["prefill_gemm"][0])
                 mat_ms.append(tm["materialize"][0])
+                rt_ms.append(tm["router"][0])
+                rs_ms.append(tm["resolve"][0])
                 n_gemm = tm["prefill_gemm"][1]
                 call_ms.append(a.elapsed_time(z))
         mf.mf_timing(ctx, [])
@@ -437,7 +439,8 @@ def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: flo
     return {"workload": f"l48e128q4 layer 0: 4096-token prefill call, hidden {H}, {E} experts, top-{k}, inter {I}, "
                         f"Q4_0, Zipf 1.2, cache {cache_pct:g}% ({plan.slots_per_layer} slots), cold",
             "tokens_per_s": round(T / (c * 1e-3), 1), "call_ms": round(c, 4), "gemm_ms": round(g, 4),
-            "gemm_waves": n_gemm, "materialize_ms": round(m, 4),
+            "gemm_waves": n_gemm, "materialize_ms": round(m, 4), "router_ms": round(statistics.mean(rt_ms), 4),
+            "resolve_ms": round(statistics.mean(rs_ms), 4),
             "materialize_gbs": round(st["bytes_materialized"] / (m * 1e-3) / 1e9, 1),
             "useful_tflops": round(useful / (g * 1e-3) / 1e12, 2),
             "roofline": {"bound": "tensor", "kernel": "prefill grouped GEMMs (gate/up+SwiGLU, down)",

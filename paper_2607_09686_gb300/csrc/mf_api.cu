@@ -86,7 +86,7 @@ struct Carve {
 
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
-  uint64_t logits, ticket, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
+  uint64_t zpart, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
   uint64_t work, err, tb_off, sx, sb, sy, sidx, sw;
   uint64_t total;
 };
@@ -104,8 +104,7 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.tr_expert = c.take<int32_t>(L * E);
   o.tr_slot = c.take<int32_t>(L * E);
   o.tr_hit = c.take<uint8_t>(L * E);
-  o.logits = c.take<float>((uint64_t)Tm * E);
-  o.ticket = c.take<unsigned>((uint64_t)Tm);
+  o.zpart = c.take<float2>(router_part_pairs(Tm, (int)E, (int)H));
   o.idx = c.take<int32_t>((uint64_t)Tm * k);
   o.g = c.take<float>((uint64_t)Tm * k);
   o.uniq = c.take<int32_t>(E);
@@ -375,8 +374,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.tr_expert = reinterpret_cast<int32_t*>(base + so.tr_expert);
   d.tr_slot = reinterpret_cast<int32_t*>(base + so.tr_slot);
   d.tr_hit = reinterpret_cast<uint8_t*>(base + so.tr_hit);
-  d.logits = reinterpret_cast<float*>(base + so.logits);
-  d.ticket = reinterpret_cast<unsigned*>(base + so.ticket);
+  d.zpart = reinterpret_cast<float2*>(base + so.zpart);
   d.idx = reinterpret_cast<int32_t*>(base + so.idx);
   d.g = reinterpret_cast<float*>(base + so.g);
   d.uniq = reinterpret_cast<int32_t*>(base + so.uniq);

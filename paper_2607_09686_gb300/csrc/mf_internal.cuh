@@ -53,8 +53,7 @@ struct Dev {
   int32_t* tr_slot;    // [L][E]
   uint8_t* tr_hit;     // [L][E]
   // per-call scratch
-  float* logits;       // [T_max][E]
-  unsigned* ticket;    // [T_max]       router last-block tickets (kept at zero between calls)
+  float2* zpart;       // router, T >= kTiledMinT: compensated logit pairs [K split][T][E]
   int32_t* idx;        // [T_max][k]
   float* g;            // [T_max][k]
   int32_t* uniq;       // [E]           distinct experts in access order
@@ -169,6 +168,10 @@ uint64_t canonical_payload_bytes(const mf_model_t& m);
 
 // kernel launchers (each returns the launch status)
 // x and bias may be pinned host memory; with x_copy, the router also writes x there (device)
+// calls with at least this many tokens take the tiled router (W_r read once per 32 tokens)
+constexpr int kTiledMinT = 16;
+// pairs of zpart the tiled router needs for any T in [kTiledMinT, T_max] (0 below that)
+size_t router_part_pairs(int T_max, int E, int H);
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
                           cudaStream_t s, float* x_copy = nullptr);
 cudaError_t launch_resolve(const Dev& d, int layer, int T, cudaStream_t s);

@@ -18,6 +18,9 @@
 // expert by counting the experts ahead of it, and keeps the k first.  With one token per call,
 // block 0 then runs the layer's slot resolve (lru_warp) on cache state it prefetched into
 // registers while the logits were being computed.  No global atomics or fences on the path.
+//
+// Calls with many tokens (T >= kTiledMinT) compute the logits as a tiled product instead, so
+// that W_r is read once per 32 tokens rather than once per token: see k_logits_tiled.
 #include <cooperative_groups.h>
 
 #include "mf_lru.cuh"
@@ -261,10 +264,224 @@ __global__ void __launch_bounds__(kThreadsR)
   }
 }
 
+
+// ---------------------------------------------------------------- many tokens per call
+// k_logits_tiled: block (expert tile, token tile, K split) computes the compensated pairs of a
+// 32-token x 64-expert tile over its range of H, from shared-memory tiles of x and W_r that
+// cp.async fills 32 columns at a time (double-buffered).  Thread (ty, tx) owns tokens 2ty, 2ty+1
+// and experts tx + 16j (j < 4).  Columns are taken two at a time with f32x2 arithmetic (the same
+// IEEE operations as dot2, on two lanes): each output keeps one compensated pair for its even
+// and one for its odd columns, added error-free at the end.  The pairs of every K split go to
+// scratch; k_topk_tiled (one warp per token) adds them in split order, rounds once, adds the
+// bias, ranks and takes the softmax exactly as the one-token path does.
+constexpr int kTT = 32, kTE = 64, kHC = 32, kThreadsT = 256;
+constexpr int kPadT = kHC + 4;  // shared row stride in floats: 16 rows read together hit 2 bank phases
+
+__device__ __forceinline__ uint64_t f2_op_add(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_op_sub(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_op_mul(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_op_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t f2_of(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ float2 f2_split(uint64_t a) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(a));
+  return make_float2(lo, hi);
+}
+
+// dot2 on two lanes: (s, c) += a * b, product split exactly by an FMA, two-sum into s
+__device__ __forceinline__ void dot2x2(uint64_t& s, uint64_t& c, uint64_t a, uint64_t b) {
+  const uint64_t p = f2_op_mul(a, b);
+  const uint64_t pe = f2_op_fma(a, b, p ^ 0x8000000080000000ull);  // a * b - p, exact
+  const uint64_t s1 = f2_op_add(s, p);
+  const uint64_t bb = f2_op_sub(s1, s);
+  const uint64_t e = f2_op_add(f2_op_sub(s, f2_op_sub(s1, bb)), f2_op_sub(p, bb));
+  s = s1;
+  c = f2_op_add(c, f2_op_add(e, pe));
+}
+
+__device__ __forceinline__ void cp_async16_zfill(void* dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src), "r"(valid ? 16 : 0)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(kThreadsT)
+    k_logits_tiled(const float* __restrict__ x, const float* __restrict__ wr, int T, int E, int H, int cps,
+                   float2* __restrict__ part) {
+  __shared__ __align__(16) float s_x[2][kTT][kPadT];
+  __shared__ __align__(16) float s_w[2][kTE][kPadT];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int e0 = (int)blockIdx.x * kTE, t0 = (int)blockIdx.y * kTT;
+  const int c0 = (int)blockIdx.z * cps, c1 = min(H / kHC, c0 + cps);
+  // one 16-byte piece of the x tile and two of the W tile per thread; rows past T or E read zeros
+  auto load = [&](int ch, int buf) {
+    {
+      const int r = tid >> 3, q = tid & 7, t = t0 + r;
+      cp_async16_zfill(&s_x[buf][r][4 * q], x + (size_t)min(t, T - 1) * H + ch * kHC + 4 * q, t < T);
+    }
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int id = tid + i * kThreadsT, r = id >> 3, q = id & 7, e = e0 + r;
+      cp_async16_zfill(&s_w[buf][r][4 * q], wr + (size_t)min(e, E - 1) * H + ch * kHC + 4 * q, e < E);
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  uint64_t S[2][4], C[2][4];  // [token][expert]: (even-column, odd-column) pairs
+#pragma unroll
+  for (int a = 0; a < 2; ++a)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) S[a][j] = C[a][j] = 0;
+  if (c0 < c1) load(c0, 0);
+  for (int ch = c0; ch < c1; ++ch) {
+    const int buf = (ch - c0) & 1;
+    if (ch + 1 < c1) {
+      load(ch + 1, buf ^ 1);  // that buffer was released by the barrier ending the previous chunk
+      asm volatile("cp.async.wait_group 1;" ::: "memory");
+    } else {
+      asm volatile("cp.async.wait_group 0;" ::: "memory");
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k4 = 0; k4 < kHC; k4 += 4) {
+      const float4 xa = *reinterpret_cast<const float4*>(&s_x[buf][2 * ty][k4]);
+      const float4 xb = *reinterpret_cast<const float4*>(&s_x[buf][2 * ty + 1][k4]);
+      const uint64_t xa01 = f2_of(xa.x, xa.y), xa23 = f2_of(xa.z, xa.w);
+      const uint64_t xb01 = f2_of(xb.x, xb.y), xb23 = f2_of(xb.z, xb.w);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 w = *reinterpret_cast<const float4*>(&s_w[buf][tx + 16 * j][k4]);
+        const uint64_t w01 = f2_of(w.x, w.y), w23 = f2_of(w.z, w.w);
+        dot2x2(S[0][j], C[0][j], w01, xa01);
+        dot2x2(S[0][j], C[0][j], w23, xa23);
+        dot2x2(S[1][j], C[1][j], w01, xb01);
+        dot2x2(S[1][j], C[1][j], w23, xb23);
+      }
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int a = 0; a < 2; ++a) {
+    const int t = t0 + 2 * ty + a;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int e = e0 + tx + 16 * j;
+      const float2 sv = f2_split(S[a][j]), cv = f2_split(C[a][j]);
+      float ss = sv.x, cc = cv.x;
+      pair_add(ss, cc, sv.y, cv.y);
+      if (t < T && e < E) part[((size_t)blockIdx.z * T + t) * E + e] = make_float2(ss, cc);
+    }
+  }
+}
+
+constexpr int kTokW = 8;  // tokens (warps) per block of k_topk_tiled
+
+__global__ void __launch_bounds__(kTokW * 32)
+    k_topk_tiled(Dev d, const float2* __restrict__ part, const float* __restrict__ bias, int T, int ks) {
+  extern __shared__ __align__(16) float s_zt[];  // [kTokW][E]
+  __shared__ int s_sel[kTokW][kMaxTopK];
+  __shared__ float s_zs[kTokW][kMaxTopK];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int t = (int)blockIdx.x * kTokW + warp;
+  if (t >= T) return;  // warp-uniform; no block-wide barrier below
+  const int E = d.E, k = d.k;
+  float* z = s_zt + (size_t)warp * E;
+  for (int e = lane; e < E; e += 32) {
+    float2 p = part[(size_t)t * E + e];
+    for (int sp = 1; sp < ks; ++sp) {
+      const float2 q = part[((size_t)sp * T + t) * E + e];
+      pair_add(p.x, p.y, q.x, q.y);
+    }
+    float v = __fadd_rn(p.x, p.y);
+    if (bias) v = __fadd_rn(v, bias[(size_t)t * E + e]);
+    z[e] = v;
+  }
+  __syncwarp();
+  for (int e = lane; e < E; e += 32) {  // rank by counting, ties to the lower id
+    const float v = z[e];
+    int r = 0;
+    for (int e2 = 0; e2 < E; ++e2) {
+      const float v2 = z[e2];
+      r += (v2 > v) || (v2 == v && e2 < e);
+    }
+    if (r < k) {
+      s_sel[warp][r] = e;
+      s_zs[warp][r] = v;
+    }
+  }
+  __syncwarp();
+  const float ex = lane < k ? expf(s_zs[warp][lane] - s_zs[warp][0]) : 0.f;
+  float den = ex;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
+  if (lane < k) {
+    d.idx[(size_t)t * k + lane] = s_sel[warp][lane];
+    d.g[(size_t)t * k + lane] = ex / den;
+  }
+}
+
+// K splits for T tokens: about kTiledBlocks blocks when the tiles alone are fewer.  A constant
+// (two blocks per SM of a 152-SM part), not the device's count, so that the planner, which runs
+// without a GPU, sizes the scratch exactly as the context does.
+constexpr int kTiledBlocks = 304;
+int tiled_splits(int T, int E, int H) {
+  const int tiles = ((T + kTT - 1) / kTT) * ((E + kTE - 1) / kTE);
+  const int nch = H / kHC;
+  int want = (kTiledBlocks + tiles - 1) / tiles;
+  if (want < 1) want = 1;
+  const int cps = (nch + want - 1) / want;
+  return (nch + cps - 1) / cps;
+}
+
+cudaError_t launch_router_tiled(const Dev& d, const float* x, const float* wr, const float* bias, int T,
+                                cudaStream_t s) {
+  const int ks = tiled_splits(T, d.E, d.H);
+  const int nch = d.H / kHC, cps = (nch + ks - 1) / ks;
+  k_logits_tiled<<<dim3((d.E + kTE - 1) / kTE, (T + kTT - 1) / kTT, ks), kThreadsT, 0, s>>>(x, wr, T, d.E, d.H, cps,
+                                                                                            d.zpart);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const size_t smem = (size_t)kTokW * d.E * sizeof(float);
+  if (smem > 48 * 1024) {
+    e = cudaFuncSetAttribute(k_topk_tiled, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  k_topk_tiled<<<(T + kTokW - 1) / kTokW, kTokW * 32, smem, s>>>(d, d.zpart, bias, T, ks);
+  return cudaGetLastError();
+}
+
 }  // namespace
+
+size_t router_part_pairs(int T_max, int E, int H) {
+  size_t most = 0;
+  for (int T = kTiledMinT; T <= T_max; ++T) {
+    const size_t n = (size_t)tiled_splits(T, E, H) * T * E;
+    if (n > most) most = n;
+  }
+  return most;
+}
 
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
                           cudaStream_t s, float* x_copy) {
+  if (T >= kTiledMinT) return launch_router_tiled(d, x, wr, bias, T, s);
   const size_t smem = (size_t)d.H * sizeof(float);
   cudaError_t e = cudaFuncSetAttribute(k_router, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
