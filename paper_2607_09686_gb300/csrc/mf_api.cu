@@ -87,7 +87,7 @@ struct Carve {
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
   uint64_t zpart, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
-  uint64_t work, err, tb_off, sx, sb, sy, sidx, sw;
+  uint64_t work, err, tb_off, sx, sb, sy, sidx, sw, stage;
   uint64_t total;
 };
 
@@ -125,6 +125,8 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.sy = c.take<float>((uint64_t)Tm * H);
   o.sidx = c.take<int32_t>((uint64_t)Tm * k);
   o.sw = c.take<float>((uint64_t)Tm * k);
+  // calls with several waves stage the next wave's misses: one payload per slot (T_max > 1)
+  o.stage = c.take<uint8_t>(Tm > 1 ? (uint64_t)S * make_layout(m).stride : 0);
   o.total = c.off;
   return o;
 }
@@ -388,6 +390,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.h = reinterpret_cast<float*>(base + so.h);
   d.part = reinterpret_cast<float*>(base + so.part);
   d.work = reinterpret_cast<unsigned*>(base + so.work);
+  d.stage = Tm > 1 ? base + so.stage : nullptr;
   d.err = reinterpret_cast<unsigned*>(base + so.err);
   d.tb_off = reinterpret_cast<int32_t*>(base + so.tb_off);
   c->stage_x = reinterpret_cast<float*>(base + so.sx);
@@ -516,16 +519,43 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   long long accesses_max = (long long)T * d.k;
   if (accesses_max > d.E) accesses_max = d.E;
   const int n_waves = (int)((accesses_max + S - 1) / S);
-  for (int w = 0; w < n_waves; ++w) {
+  // Materialisation on the side stream.  One wave: its misses straight into their slots, then
+  // the compute.  Several waves: wave 0 as above; wave w + 1's misses are staged while wave w
+  // computes (their slots may still be read by it) and committed to the slots once it is done.
+  const bool staged = n_waves > 1 && d.stage;
+  auto wave_width = [&](int w) {
     long long width = accesses_max - (long long)w * S;
-    if (width > S) width = S;
-    MF_CUDA(cudaEventRecord(c->ev_fork[w], s));
-    MF_CUDA(cudaStreamWaitEvent(c->side, c->ev_fork[w], 0));
+    return (int)(width > S ? S : width);
+  };
+  MF_CUDA(cudaEventRecord(c->ev_fork[0], s));
+  MF_CUDA(cudaStreamWaitEvent(c->side, c->ev_fork[0], 0));
+  timer_mark(c, kTMaterialize, 0, c->side);
+  MF_CUDA(launch_materialize(d, layer, 0, wave_width(0), c->side));
+  timer_mark(c, kTMaterialize, 1, c->side);
+  MF_CUDA(cudaEventRecord(c->ev_join[0], c->side));
+  auto stage_next = [&](int w) -> cudaError_t {  // side stream: wave w's misses into the stage
     timer_mark(c, kTMaterialize, 0, c->side);
-    MF_CUDA(launch_materialize(d, layer, w, (int)width, c->side));
+    cudaError_t e = launch_materialize(d, layer, w, wave_width(w), c->side, d.stage);
     timer_mark(c, kTMaterialize, 1, c->side);
-    MF_CUDA(cudaEventRecord(c->ev_join[w], c->side));
-    MF_CUDA(cudaStreamWaitEvent(s, c->ev_join[w], 0));
+    return e;
+  };
+  if (staged) MF_CUDA(stage_next(1));
+  for (int w = 0; w < n_waves; ++w) {
+    const int width = wave_width(w);
+    if (w > 0) {  // side stream, once wave w - 1 has computed: wave w's misses into their slots
+      MF_CUDA(cudaEventRecord(c->ev_fork[w], s));
+      MF_CUDA(cudaStreamWaitEvent(c->side, c->ev_fork[w], 0));
+      if (staged) {
+        MF_CUDA(launch_stage_commit(d, layer, w, d.stage, c->side));
+      } else {
+        timer_mark(c, kTMaterialize, 0, c->side);
+        MF_CUDA(launch_materialize(d, layer, w, width, c->side));
+        timer_mark(c, kTMaterialize, 1, c->side);
+      }
+      MF_CUDA(cudaEventRecord(c->ev_join[w], c->side));
+      if (staged && w + 1 < n_waves) MF_CUDA(stage_next(w + 1));  // overlaps wave w's compute
+    }
+    MF_CUDA(cudaStreamWaitEvent(s, c->ev_join[w], 0));  // wave w's experts are in their slots
     if (gemm) {
       timer_mark(c, kTPrefill, 0, s);
       MF_CUDA(launch_prefill_gateup(d, c->tm_gu, layer, w, s));

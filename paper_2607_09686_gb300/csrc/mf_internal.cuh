@@ -71,6 +71,7 @@ struct Dev {
   // per 128-assignment block t and K step kk of 32: [bf16 hi 8 KiB | bf16 lo 8 KiB]
   uint8_t* xt;         // x tiles:  t * (H / 32) + kk
   uint8_t* ht;         // h tiles:  t * (I / 32) + kk
+  uint8_t* stage;      // [S_alloc] payloads: a wave's misses staged while the previous wave computes (T_max > 1)
   unsigned* work;      // [4]           arrival counter (64-bit) of the fused one-token FFN kernel
   unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
 };
@@ -175,7 +176,11 @@ size_t router_part_pairs(int T_max, int E, int H);
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
                           cudaStream_t s, float* x_copy = nullptr);
 cudaError_t launch_resolve(const Dev& d, int layer, int T, cudaStream_t s);
-cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s);
+// dst_stage null: each miss into its slot; else miss m of the wave to dst_stage + m * stride
+cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s,
+                               uint8_t* dst_stage = nullptr);
+// the wave's staged payloads into their slots
+cudaError_t launch_stage_commit(const Dev& d, int layer, int wave, const uint8_t* stage, cudaStream_t s);
 cudaError_t launch_gateup(const Dev& d, int layer, int wave, int wave_width, const float* x, cudaStream_t s);
 cudaError_t launch_down_single(const Dev& d, int layer, float* y, cudaStream_t s);
 cudaError_t launch_down_partial(const Dev& d, int layer, int wave, int wave_width, cudaStream_t s);

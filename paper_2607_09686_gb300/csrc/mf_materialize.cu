@@ -4,23 +4,35 @@
 // The misses are decided on the device (slot resolve), so the copy is driven by the GPU
 // itself: SMs load 16-byte vectors straight from the pinned, device-mapped pack over the
 // CPU-GPU link and store them into the slot, with no host round trip.  Launched on the
-// context's side stream: two blocks per SM stride over each missed payload of the wave in
-// turn; with no miss every block returns at once.
+// context's side stream: one small block per SM (two warps, 8 KB of loads in flight each: the
+// link saturates at a fraction of that) strides over each missed payload of the wave in turn;
+// with no miss every block returns at once.  Both kernels here ask
+// for the largest shared-memory carveout although they use none: an SM runs blocks of one
+// carveout at a time, so only then can they share SMs with a running expert-FFN kernel (which
+// needs most of the shared memory) instead of holding those SMs until they finish.
+//
+// Calls with several waves stage the misses of wave w + 1 (one payload per miss, in miss
+// order) while wave w computes: the slots they go to may still be read by wave w.  Once wave w
+// is done, k_stage_commit copies the staged payloads HBM -> HBM into their slots.
 #include "mf_internal.cuh"
 
 namespace mf {
 namespace {
 
 constexpr int kUnroll = 8;
+constexpr int kMatThreads = 64;
 
-__global__ void __launch_bounds__(256) k_materialize(Dev d, int layer, int wave) {
+// dst_stage: null to write each miss into its slot, else miss m of the wave goes to
+// dst_stage + m * stride
+__global__ void __launch_bounds__(kMatThreads) k_materialize(Dev d, int layer, int wave, uint8_t* dst_stage) {
   const int n_miss = d.info[2 + wave];
   const size_t nvec = d.lay.stride / 16;  // 16-byte vectors per payload
   const size_t step = (size_t)gridDim.x * blockDim.x * kUnroll;
   for (int m = 0; m < n_miss; ++m) {
     const int u = d.miss_list[wave * d.S_active + m];
     const uint4* src = reinterpret_cast<const uint4*>(d.pack + ((size_t)layer * d.E + d.uniq[u]) * d.lay.stride);
-    uint4* dst = reinterpret_cast<uint4*>(d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride);
+    uint4* dst = reinterpret_cast<uint4*>(dst_stage ? dst_stage + (size_t)m * d.lay.stride
+                                                    : d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride);
     for (size_t i0 = (size_t)blockIdx.x * blockDim.x * kUnroll + threadIdx.x; i0 < nvec; i0 += step) {
       uint4 v[kUnroll];
 #pragma unroll
@@ -37,19 +49,68 @@ __global__ void __launch_bounds__(256) k_materialize(Dev d, int layer, int wave)
   }
 }
 
-}  // namespace
+// the wave's staged payloads into their slots (HBM -> HBM)
+__global__ void __launch_bounds__(256) k_stage_commit(Dev d, int layer, int wave, const uint8_t* __restrict__ stage) {
+  const int n_miss = d.info[2 + wave];
+  const size_t nvec = d.lay.stride / 16;
+  const size_t step = (size_t)gridDim.x * blockDim.x * 4;
+  for (int m = 0; m < n_miss; ++m) {
+    const int u = d.miss_list[wave * d.S_active + m];
+    const uint4* src = reinterpret_cast<const uint4*>(stage + (size_t)m * d.lay.stride);
+    uint4* dst = reinterpret_cast<uint4*>(d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride);
+    for (size_t i0 = (size_t)blockIdx.x * blockDim.x * 4 + threadIdx.x; i0 < nvec; i0 += step) {
+      uint4 v[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const size_t i = i0 + (size_t)r * blockDim.x;
+        if (i < nvec) v[r] = src[i];
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        const size_t i = i0 + (size_t)r * blockDim.x;
+        if (i < nvec) dst[i] = v[r];
+      }
+    }
+  }
+}
 
-cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s) {
-  if (max_miss <= 0) return cudaSuccess;
-  static int n_sm = 0;
-  if (!n_sm) {
+int n_sm() {
+  static int n = 0;
+  if (!n) {
     int dev = 0;
     cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-    if (n_sm <= 0) n_sm = 1;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 1;
   }
-  // two blocks per SM stream all misses of the wave; the CPU-GPU link saturates well below this
-  k_materialize<<<2 * n_sm, 256, 0, s>>>(d, layer, wave);
+  return n;
+}
+
+}  // namespace
+
+cudaError_t max_shared_carveout() {
+  static cudaError_t e = [] {
+    cudaError_t r = cudaFuncSetAttribute(k_materialize, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                         cudaSharedmemCarveoutMaxShared);
+    if (r == cudaSuccess)
+      r = cudaFuncSetAttribute(k_stage_commit, cudaFuncAttributePreferredSharedMemoryCarveout,
+                               cudaSharedmemCarveoutMaxShared);
+    return r;
+  }();
+  return e;
+}
+
+cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s, uint8_t* dst_stage) {
+  if (max_miss <= 0) return cudaSuccess;
+  cudaError_t e = max_shared_carveout();
+  if (e != cudaSuccess) return e;
+  k_materialize<<<n_sm(), kMatThreads, 0, s>>>(d, layer, wave, dst_stage);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_stage_commit(const Dev& d, int layer, int wave, const uint8_t* stage, cudaStream_t s) {
+  cudaError_t e = max_shared_carveout();
+  if (e != cudaSuccess) return e;
+  k_stage_commit<<<2 * n_sm(), 256, 0, s>>>(d, layer, wave, stage);
   return cudaGetLastError();
 }
 
