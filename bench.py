@@ -35,7 +35,7 @@ N_TOKENS = 256
 # DRAM bytes (read + write) of one launch of the roofline kernel (the fused one-token FFN) from
 # the ncu capture summarised under profiles/, valid while the kernel sources hash to `sha`
 # (otherwise the line reports null: the counters no longer describe the kernel that ran).
-KERNEL_TRAFFIC = {"sha": "3e610f36a78815b0", "bytes": 40194816,
+KERNEL_TRAFFIC = {"sha": "6f6f9a29fd6e3efc", "bytes": 40196096,
                   "files": ("paper_2607_09686_gb300/csrc/mf_decode.cu", "paper_2607_09686_gb300/csrc/mf_dequant.cuh",
                             "paper_2607_09686_gb300/csrc/mf_internal.cuh")}
 
@@ -384,7 +384,31 @@ def resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, s
     gbs = bytes_per_launch / (us * 1e-6) / 1e9
     return {"achieved": round(gbs, 1), "frac": round(gbs / hbm, 4), "us_per_launch": round(us, 3), "launches": n,
             "misses_in_timed_replays": st["misses"],
-            "how": "same calls, 100 % cache warmed by two passes (every launch all-resident), L2 flushed per replay"}
+            "how": "same calls, 100 % cache warmed by two passes (every launch all-resident), L2 flushed per replay",
+            "read_floor": read_floor(torch, device, stream, flush, bytes_per_launch, hbm)}
+
+
+def read_floor(torch, device, stream, flush, nbytes, hbm, reps: int = 20) -> dict:
+    """What one read-only launch of the same size achieves: a torch.sum over nbytes of fp32 from a
+    cold L2, CUDA events around the launch (the launch and first-access latency that bound any
+    single kernel of this size)."""
+    buf = torch.ones(nbytes // 4, dtype=torch.float32, device=device)
+    out = torch.empty((), dtype=torch.float32, device=device)
+    times = []
+    with torch.cuda.stream(stream):
+        for i in range(3 + reps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            torch.sum(buf, dtype=torch.float32, out=out)
+            b.record(stream)
+            b.synchronize()
+            if i >= 3:
+                times.append(a.elapsed_time(b) * 1e3)
+    us = statistics.mean(times)
+    gbs = nbytes / (us * 1e-6) / 1e9
+    return {"us": round(us, 3), "achieved": round(gbs, 1), "frac": round(gbs / hbm, 4),
+            "how": "one torch.sum launch over the same bytes after an L2 flush, CUDA events around it"}
 
 
 def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: float = 15.0) -> dict:

@@ -427,7 +427,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
     return rc;
   }
   size_t smem = resolve_smem_bytes(d);
-  if (smem > 48 * 1024) {
+  if (smem > 232448) {  // the resolve kernel's shared memory (at most 1024 experts and slots: 144 KB)
     free_ctx(c);
     return MF_E_INVAL;
   }
@@ -505,7 +505,6 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   }
 
   const bool gemm = T > 1 && c->prefill_min_t > 0 && T >= c->prefill_min_t;
-  if (gemm) MF_CUDA(launch_tile_x(d, x, T, s));
 
   if (T == 1 && c->ffn_fused) {  // one launch: expert FFN, with the misses materialised inside
     timer_mark(c, kTFfn, 0, s);
@@ -533,6 +532,7 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   MF_CUDA(launch_materialize(d, layer, 0, wave_width(0), c->side));
   timer_mark(c, kTMaterialize, 1, c->side);
   MF_CUDA(cudaEventRecord(c->ev_join[0], c->side));
+  if (gemm) MF_CUDA(launch_tile_x(d, x, T, s));  // the GEMM's x tiles, while wave 0 materialises
   auto stage_next = [&](int w) -> cudaError_t {  // side stream: wave w's misses into the stage
     timer_mark(c, kTMaterialize, 0, c->side);
     cudaError_t e = launch_materialize(d, layer, w, wave_width(w), c->side, d.stage);

@@ -1,4 +1,5 @@
-"""One 4096-token Q4_0 call (hidden 2048, 128 experts, top-8, inter 768), 1 layer, all slots."""
+"""One 4096-token Q4_0 call (hidden 2048, 128 experts, top-8, inter 768), 1 layer, from a cold
+cache, twice.  Argument: slots per layer (default 128: every expert resident, one wave)."""
 import sys
 sys.path[:0] = [".", "tests"]
 import torch, synth
@@ -7,7 +8,8 @@ import paper_2607_09686_gb300 as mf
 cfg = synth.CONFIGS["l48e128q4"]
 T = 4096
 shape = Shape(1, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype)
-ctx = Ctx(shape, 128, max_tokens=T, workers=16)
+slots = int(sys.argv[1]) if len(sys.argv) > 1 else 128
+ctx = Ctx(shape, slots, max_tokens=T, workers=16)
 r = synth.routes(0, 0, 0, 128, 8, T, 1.2, 0.0)
 x = torch.from_numpy(synth.activations(0, 0, 0, 0, T, cfg.hidden)).cuda()
 b = torch.from_numpy(synth.plant_bias(r, 128)).cuda()
