@@ -400,7 +400,7 @@ def read_floor(torch, device, stream, flush, nbytes, hbm, reps: int = 20) -> dic
             flush.zero_()
             a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             a.record(stream)
-            torch.sum(buf, dtype=torch.float32, out=out)
+            torch.sum(buf, 0, dtype=torch.float32, out=out)
             b.record(stream)
             b.synchronize()
             if i >= 3:

@@ -323,22 +323,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 // their gate/up items, publish it, meet every other block at a grid-wide arrival counter (bounded
 // wait), and then take the down items with the k experts' h.  The counter never resets: each launch adds one
 // arrival per block, and a block waits for the multiple of gridDim.x that completes its launch.
-// One item of a missed expert, by the whole warp: `bytes` (a multiple of 16) from the pinned pack
-// into the shared-memory stage, every piece in flight at once (cp.async); then lane 0 writes the
-// stage through to the expert's HBM slot with one bulk copy (completion awaited before the stage
-// is refilled and before the block exits).
-__device__ __forceinline__ void host_fill(unsigned char* stage, uint8_t* slot, const uint8_t* pack, uint32_t bytes,
-                                          int lane) {
+// Missed experts' bytes, by the whole warp: host_pull issues `bytes` (a multiple of 16) from the
+// pinned pack into shared memory as 16-byte cp.async pieces (every piece in flight at once; the
+// caller commits and waits); once they have landed, slot_write_through makes the warp's
+// writes visible to the async proxy and lane 0 writes the buffer through to the expert's HBM
+// slot with one bulk copy (completion awaited before the buffer is refilled and before the
+// block exits).
+__device__ __forceinline__ void host_pull(unsigned char* dst, const uint8_t* pack, uint32_t bytes, int lane) {
   const int n = (int)(bytes / 16);
   for (int i = lane; i < n; i += 32)
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(stage + (size_t)i * 16)),
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst + (size_t)i * 16)),
                  "l"(pack + (size_t)i * 16)
                  : "memory");
-  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+__device__ __forceinline__ void slot_write_through(unsigned char* src, uint8_t* slot, uint32_t bytes, int lane) {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // before the bulk copy reads them
   __syncwarp();
   if (lane == 0) {
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(slot), "r"(smem_u32(stage)),
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(slot), "r"(smem_u32(src)),
                  "r"(bytes)
                  : "memory");
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
@@ -484,38 +486,61 @@ __global__ void __launch_bounds__(kThreadsF, 1)
           if (!s_miss[j] && !mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
     }
   } else if (warp == kConsumers + 1) {
-    // ---- link warp: the missed experts' items through ring B, then their down records
-    Ring ring;
+    // ---- link warp: the missed experts' items through ring B (both stages in flight at once),
+    // then all their down records at once (after the items: the grid barrier and the h split
+    // overlap that transfer)
     bool ok = true;
-    const int R = cg.R, nrb = d.I / R;
+    const int R = cg.R, nrb = d.I / R, n_li = mine_g - nres;
     const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
     const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
     const size_t doff = (size_t)r0 * d.lay.rs_d;
-    for (int t = nres, it = 0; t < mine_g; ++t, ++it) {
-      if (it >= NB) {
+    auto issue_item = [&](int t, int s) {  // the block's link item t into ring B stage s: one group
+      const int item = s_gord[nres + t], u = item / nrb, rb = item % nrb;
+      const size_t off = (size_t)rb * R * rs;
+      host_pull(sm.stage0 + (size_t)(NA + s) * f.stage_bytes, s_hgu[u] + off, bytes, lane);
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+    int issued = 0;
+    for (; issued < n_li && issued < NB; ++issued) issue_item(issued, issued);
+    for (int t = 0; t < n_li; ++t) {
+      const int s = t % NB;
+      if (issued > t + 1)  // item t's group is complete once at most the later one is pending
+        asm volatile("cp.async.wait_group 1;" ::: "memory");
+      else
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+      const int item = s_gord[nres + t], u = item / nrb, rb = item % nrb;
+      slot_write_through(sm.stage0 + (size_t)(NA + s) * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, lane);
+      if (lane == 0) mbar_arrive(&sm.full[NA + s]);  // release: every lane's stage writes
+      if (issued < n_li) {  // refill the stage once the consumers are done with item t
         int w = 1;
         if (lane == 0) {
-          w = mbar_wait(&sm.empty[NA + ring.s], ring.phase ^ 1u);
-          slot_writes_read();  // the stage's previous write-through has read it
+          w = mbar_wait(&sm.empty[NA + s], (uint32_t)(t / NB) & 1u);
+          slot_writes_read();  // and its write-through has read it
         }
         if (!__shfl_sync(0xffffffffu, w, 0)) {
           ok = false;
           break;
         }
+        issue_item(issued, s);
+        ++issued;
       }
-      const int item = s_gord[t], u = item / nrb, rb = item % nrb;
-      const size_t off = (size_t)rb * R * rs;
-      host_fill(sm.stage0 + (size_t)(NA + ring.s) * f.stage_bytes, s_gu[u] + off, s_hgu[u] + off, bytes,
-                lane);                                      // ends with a warp barrier
-      if (lane == 0) mbar_arrive(&sm.full[NA + ring.s]);  // release: every lane's stage writes
-      ring.next(NB);
     }
-    if (ok)
+    if (ok) {
+      bool any = false;
       for (int j = 0; j < mine_d; ++j)
         if (s_miss[j]) {
-          host_fill(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, s_hgu[j] + d.lay.d_off + doff, dbytes, lane);
-          if (lane == 0) mbar_arrive(&full_d[j]);
+          host_pull(dbuf + (size_t)j * f.dn_bytes, s_hgu[j] + d.lay.d_off + doff, dbytes, lane);
+          any = true;
         }
+      if (any) {
+        asm volatile("cp.async.wait_all;" ::: "memory");
+        for (int j = 0; j < mine_d; ++j)
+          if (s_miss[j]) {
+            slot_write_through(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, dbytes, lane);
+            if (lane == 0) mbar_arrive(&full_d[j]);
+          }
+      }
+    }
     if (lane == 0) {
       if (!ok) atomicExch(d.err, 1u);
       slot_writes_done();  // every write-through complete before the block exits
