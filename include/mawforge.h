@@ -52,6 +52,10 @@ extern "C" {
 #define MF_Q4_0 2
 #define MF_Q8_0 8
 
+/* Access orders of a step with several tokens (mf_access_order). */
+#define MF_ORDER_FIRST_OCCURRENCE 0 /* distinct experts in (token, rank) first-occurrence order */
+#define MF_ORDER_RESIDENT_FIRST 1   /* the experts resident when the step starts first, then the rest */
+
 /* Shape of the routed-expert part of a model.  Each expert is a SwiGLU FFN with separate
  * gate [inter x hidden], up [inter x hidden] and down [hidden x inter] tensors.
  * Requirements: hidden and inter multiples of 32; 1 <= top_k <= 8; top_k <= n_experts <= 1024. */
@@ -147,6 +151,18 @@ int mf_moe_forward(mf_ctx_t* ctx, int layer, const float* x, const float* router
  * if that fails; MF_E_CUDA if the driver cannot describe the slot pool to the copy engine).
  * Host only; applies to calls issued afterwards. */
 int mf_prefill_threshold(mf_ctx_t* ctx, int min_tokens);
+
+/* Order in which a call with T > 1 presents its distinct experts to the layer's cache
+ * (section "Native Serving Path": the cache is consulted per routed expert; the paper does not
+ * order a batched step's accesses).  MF_ORDER_FIRST_OCCURRENCE (the default): (token, rank)
+ * first-occurrence order.  MF_ORDER_RESIDENT_FIRST: the experts that are resident when the
+ * call starts come first (in first-occurrence order among themselves), then the others (in
+ * first-occurrence order): every one of them hits, whereas in first-occurrence order an early
+ * miss can evict an expert the same step needs later.  Calls with T = 1 are unaffected (their k
+ * distinct experts form one wave, and no access of a wave evicts another of it).  Waves,
+ * counters, traces and outputs follow the chosen order.  MF_E_INVAL for any other value.  Host
+ * only; applies to calls issued afterwards. */
+int mf_access_order(mf_ctx_t* ctx, int order);
 
 /* As mf_moe_forward, with x, logit_bias, y, idx_out and w_out in HOST memory.  Pageable
  * buffers: x and the bias are staged into the context's device buffers and the outputs copied

@@ -57,7 +57,7 @@ def _lib():
         lib.orc_lru_free.restype = None
         lib.orc_lru_free.argtypes = [vp]
         lib.orc_lru_step.restype = i32
-        lib.orc_lru_step.argtypes = [vp, vp, i32, i32, vp, vp, vp]
+        lib.orc_lru_step.argtypes = [vp, vp, i32, i32, i32, vp, vp, vp]
         lib.orc_lru_stats.restype = None
         lib.orc_lru_stats.argtypes = [vp, vp]
         lib.orc_lru_occupancy.restype = i32
@@ -154,17 +154,18 @@ class LRU:
             _lib().orc_lru_free(h)
             self._h = None
 
-    def step(self, idx: np.ndarray):
-        """Process one step's routes [T,k]: returns (experts, slots, hits) of its accesses."""
+    def step(self, idx: np.ndarray, order: int = 0):
+        """Process one step's routes [T,k]: returns (experts, slots, hits) of its accesses.
+        order 0: first-occurrence order; 1: for T > 1, the experts resident at the start first."""
         idx = np.ascontiguousarray(idx, dtype=np.int32)
         T, k = idx.reshape(-1, idx.shape[-1]).shape
         n = T * k
         uniq = np.empty(n, np.int32)
         slot = np.empty(n, np.int32)
         hit = np.empty(n, np.uint8)
-        U = _lib().orc_lru_step(self._h, _ptr(idx), T, k, _ptr(uniq), _ptr(slot), _ptr(hit))
+        U = _lib().orc_lru_step(self._h, _ptr(idx), T, k, int(order), _ptr(uniq), _ptr(slot), _ptr(hit))
         if U < 0:
-            raise ValueError("expert id out of range")
+            raise ValueError("expert id out of range" if U == -1 else "out of memory")
         return uniq[:U].copy(), slot[:U].copy(), hit[:U].astype(bool)
 
     def stats(self) -> dict:

@@ -228,10 +228,12 @@ orc_lru* orc_lru_new(int E, int S, uint64_t payload) {
 }
 
 /* One step: the step's accesses are its distinct experts in (token, rank) first-occurrence
- * order.  Each access: resident -> hit; else miss into the lowest free slot, or, with no
- * free slot, into the slot of the least recently used expert, which is evicted.
+ * order; with order 1 and T > 1, the experts resident when the step starts come first (in
+ * that order among themselves), then the others (likewise).  Each access: resident -> hit;
+ * else miss into the lowest free slot, or, with no free slot, into the slot of the least
+ * recently used expert, which is evicted.
  * Writes the access list (expert, slot after the access, hit bit); returns its length. */
-int orc_lru_step(orc_lru* c, const int32_t* idx, int T, int k, int32_t* uniq, int32_t* slot,
+int orc_lru_step(orc_lru* c, const int32_t* idx, int T, int k, int order, int32_t* uniq, int32_t* slot,
                  uint8_t* hit) {
   int U = 0;
   for (int p = 0; p < T * k; ++p) {
@@ -240,6 +242,17 @@ int orc_lru_step(orc_lru* c, const int32_t* idx, int T, int k, int32_t* uniq, in
     for (int u = 0; u < U; ++u)
       if (uniq[u] == e) seen = 1;
     if (!seen) uniq[U++] = e;
+  }
+  if (order == 1 && T > 1) { /* resident ones first, each group keeping its order */
+    int32_t* first = (int32_t*)malloc(sizeof(int32_t) * (size_t)(U > 0 ? U : 1));
+    if (!first) return -2;
+    int n = 0;
+    for (int u = 0; u < U; ++u)
+      if (c->slot_of[uniq[u]] >= 0) first[n++] = uniq[u];
+    for (int u = 0; u < U; ++u)
+      if (c->slot_of[uniq[u]] < 0) first[n++] = uniq[u];
+    memcpy(uniq, first, sizeof(int32_t) * (size_t)U);
+    free(first);
   }
   for (int u = 0; u < U; ++u) {
     int e = uniq[u], s = c->slot_of[e];

@@ -17,7 +17,7 @@ import os
 __all__ = [
     "MFError", "Model", "PlanReq", "Plan", "Stats", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
     "mf_payload_bytes", "mf_plan", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
-    "mf_moe_forward_host", "mf_prefill_threshold", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_expert_ffn_noalloc", "mf_destroy",
+    "mf_moe_forward_host", "mf_prefill_threshold", "mf_access_order", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_expert_ffn_noalloc", "mf_destroy",
     "mf_strerror", "mf_last_cuda_error",
 ]
 
@@ -71,6 +71,7 @@ _sig = {
     "mf_moe_forward": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp]),
     "mf_moe_forward_host": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp]),
     "mf_prefill_threshold": (_i32, [_vp, _i32]),
+    "mf_access_order": (_i32, [_vp, _i32]),
     "mf_stats": (_i32, [_vp, _i32, ctypes.POINTER(Stats), _i32]),
     "mf_reset": (_i32, [_vp, _i32, _vp]),
     "mf_trace": (_i32, [_vp, _i32, _vp, _vp, _vp, _i32, ctypes.POINTER(_i32)]),
@@ -181,6 +182,15 @@ def mf_moe_forward_host(ctx: int, layer: int, x, router_w, logit_bias, T: int, y
 def mf_prefill_threshold(ctx: int, min_tokens: int) -> None:
     """Calls with T >= min_tokens use the tensor-core grouped GEMMs (0 = never)."""
     _check(_lib.mf_prefill_threshold(ctx, min_tokens), "mf_prefill_threshold")
+
+
+MF_ORDER_FIRST_OCCURRENCE = 0
+MF_ORDER_RESIDENT_FIRST = 1
+
+
+def mf_access_order(ctx: int, order: int) -> None:
+    """Order of a many-token call's accesses to the cache (MF_ORDER_*)."""
+    _check(_lib.mf_access_order(ctx, order), "mf_access_order")
 
 
 def mf_stats(ctx: int, layer: int = -1, reset: bool = False) -> dict:

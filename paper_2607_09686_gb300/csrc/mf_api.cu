@@ -326,6 +326,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.S_alloc = S;
   d.S_active = S;
   d.T_max = Tm;
+  d.order = MF_ORDER_FIRST_OCCURRENCE;
   d.lay = make_layout(*m);
 
   int rc = MF_OK;
@@ -529,13 +530,13 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   MF_CUDA(cudaEventRecord(c->ev_fork[0], s));
   MF_CUDA(cudaStreamWaitEvent(c->side, c->ev_fork[0], 0));
   timer_mark(c, kTMaterialize, 0, c->side);
-  MF_CUDA(launch_materialize(d, layer, 0, wave_width(0), c->side));
+  MF_CUDA(launch_materialize(d, layer, 0, wave_width(0), c->side, nullptr, gemm));
   timer_mark(c, kTMaterialize, 1, c->side);
   MF_CUDA(cudaEventRecord(c->ev_join[0], c->side));
   if (gemm) MF_CUDA(launch_tile_x(d, x, T, s));  // the GEMM's x tiles, while wave 0 materialises
   auto stage_next = [&](int w) -> cudaError_t {  // side stream: wave w's misses into the stage
     timer_mark(c, kTMaterialize, 0, c->side);
-    cudaError_t e = launch_materialize(d, layer, w, wave_width(w), c->side, d.stage);
+    cudaError_t e = launch_materialize(d, layer, w, wave_width(w), c->side, d.stage, gemm);
     timer_mark(c, kTMaterialize, 1, c->side);
     return e;
   };
@@ -549,7 +550,7 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
         MF_CUDA(launch_stage_commit(d, layer, w, d.stage, c->side));
       } else {
         timer_mark(c, kTMaterialize, 0, c->side);
-        MF_CUDA(launch_materialize(d, layer, w, width, c->side));
+        MF_CUDA(launch_materialize(d, layer, w, width, c->side, nullptr, gemm));
         timer_mark(c, kTMaterialize, 1, c->side);
       }
       MF_CUDA(cudaEventRecord(c->ev_join[w], c->side));
@@ -601,6 +602,12 @@ int mf_prefill_threshold(mf_ctx_t* c, int min_tokens) {
     if (rc) return rc;
   }
   c->prefill_min_t = min_tokens;
+  return MF_OK;
+}
+
+int mf_access_order(mf_ctx_t* c, int order) {
+  if (!c || (order != MF_ORDER_FIRST_OCCURRENCE && order != MF_ORDER_RESIDENT_FIRST)) return MF_E_INVAL;
+  c->d.order = order;
   return MF_OK;
 }
 

@@ -8,7 +8,10 @@
 //
 // One warp per weight row.  Each lane holds whole 16-byte vectors of the row's codes in
 // registers (Q8_0: 16 weights, Q4_0: one 32-weight block) and reuses them for every token
-// the expert serves.  Codes are turned into floats exactly by placing each byte (or
+// the expert serves.  The down projection of a call with several tokens runs 8 or 16 rows per
+// block and stages the h vectors of up to kChunkT of the expert's assignments at a time in
+// shared memory, arranged so that the lanes' loads of one vector part are contiguous, for all
+// its rows to read.  Codes are turned into floats exactly by placing each byte (or
 // nibble) in the low mantissa bits of 2^23 with a byte permute and subtracting 2^23 plus
 // the code offset (the int8 -> float "magic number" conversion of Kim et al., "Who says
 // elephants can't run", 2022), which costs one PRMT and one FADD per weight instead of an
@@ -23,6 +26,42 @@ using namespace dq;
 
 __device__ __forceinline__ const uint8_t* slot_base(const Dev& d, int layer, int slot) {
   return d.pool + ((size_t)layer * d.S_alloc + slot) * d.lay.stride;
+}
+
+// rows (warps) per block of the many-token kernels: 16 where the row's registers fit in 128 per
+// thread, else 8
+template <int QT, int VPL>
+__host__ __device__ constexpr int rows_per_block() {
+  return (QT == kQ8 && (VPL <= 3 || VPL == 6)) ? 16 : 8;
+}
+constexpr int kChunkT = 8;           // tokens whose activations are staged at once
+constexpr int kStageFloats = 24576;  // at most 96 KB of staged activations
+
+// Shared-memory order of a staged vector of n floats (n = nvec * kW): float4 j of vector v at
+// float4 index j * nvec + v, so that lane-consecutive vectors v read consecutive float4s.
+template <int QT>
+__device__ __forceinline__ void stage_vec(float4* dst, const float* __restrict__ src, int nvec) {
+  constexpr int kP = Vec<QT>::kW / 4;  // float4 parts per vector
+  for (int q = threadIdx.x; q < nvec * kP; q += blockDim.x) {
+    const float4 f = __ldg(reinterpret_cast<const float4*>(src) + q);
+    dst[(q % kP) * nvec + q / kP] = f;
+  }
+}
+template <int QT>
+__device__ __forceinline__ XV<QT> staged_x(const float4* xs, int nvec, int v) {
+  XV<QT> r;
+#pragma unroll
+  for (int j = 0; j < Vec<QT>::kW / 4; ++j) {
+    const float4 f = xs[j * nvec + v];
+    r.p[2 * j] = f2_pack(__float_as_uint(f.x), __float_as_uint(f.y));
+    r.p[2 * j + 1] = f2_pack(__float_as_uint(f.z), __float_as_uint(f.w));
+  }
+  return r;
+}
+// tokens staged per chunk for vectors of n floats
+__host__ __device__ __forceinline__ int chunk_tokens(int n) {
+  const int c = kStageFloats / n;
+  return c < 1 ? 1 : (c > kChunkT ? kChunkT : c);
 }
 
 // ---------------------------------------------------------------- gate/up + SwiGLU
@@ -122,40 +161,48 @@ __global__ void __launch_bounds__(256) k_down_single(Dev d, int layer, float* __
 }
 
 // ---------------------------------------------------------------- down, per assignment (T > 1)
-// grid (ceil(H / 8), wave width): part[t*k+j][c] = sum_r Wd[c,r] h[t*k+j][r]
+// grid (ceil(H / RB), wave width): part[t*k+j][c] = sum_r Wd[c,r] h[t*k+j][r]; h of the
+// expert's assignments staged chunk by chunk.
 template <int QT, int VPL>
-__global__ void __launch_bounds__(256) k_down_partial(Dev d, int layer, int wave) {
+__global__ void __launch_bounds__(rows_per_block<QT, VPL>() * 32, 1) k_down_partial(Dev d, int layer, int wave) {
+  extern __shared__ float4 s_hs[];  // [chunk][I / 4] in staged order
   const int u = wave * d.S_active + blockIdx.y;
-  if (u >= d.info[0]) return;
+  if (u >= d.info[0]) return;  // block-uniform
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int c = blockIdx.x * 8 + warp;
-  if (c >= d.H) return;
+  const int c = blockIdx.x * rows_per_block<QT, VPL>() + warp;
+  const bool row_ok = c < d.H;
   const uint8_t* slot = slot_base(d, layer, d.uslot[u]);
-  const uint8_t* q = slot + d.lay.d_off + (size_t)c * d.lay.rs_d;
+  const uint8_t* q = slot + d.lay.d_off + (size_t)(row_ok ? c : 0) * d.lay.rs_d;
   const __half* s = reinterpret_cast<const __half*>(q + d.lay.o_ds);
-  const int nvec = d.lay.qrow_d / 16;
+  const int nvec = d.lay.qrow_d / 16, I = d.I, nq = I / 4;
   uint4 w[VPL];
   float sc[VPL];
 #pragma unroll
   for (int i = 0; i < VPL; ++i) {
     const int v = lane + 32 * i;
-    if (v < nvec) {
+    if (row_ok && v < nvec) {
       w[i] = ld_stream(q + 16 * v);
       sc[i] = __half2float(s[scale_index<QT>(v)]);
     }
   }
-  const int a0 = d.asg_off[u], a1 = d.asg_off[u + 1];
-  for (int a = a0; a < a1; ++a) {
-    const int pos = d.asg[a];
-    const float* hp = d.h + (size_t)pos * d.I;
-    float part = 0.f;
+  const int a0 = d.asg_off[u], a1 = d.asg_off[u + 1], ct = chunk_tokens(I);
+  for (int c0 = a0; c0 < a1; c0 += ct) {
+    const int n = min(ct, a1 - c0);
+    __syncthreads();
+    for (int t = 0; t < n; ++t) stage_vec<QT>(s_hs + (size_t)t * nq, d.h + (size_t)d.asg[c0 + t] * I, nvec);
+    __syncthreads();
+    if (!row_ok) continue;
+    for (int t = 0; t < n; ++t) {
+      const float4* hs = s_hs + (size_t)t * nq;
+      float part = 0.f;
 #pragma unroll
-    for (int i = 0; i < VPL; ++i) {
-      const int v = lane + 32 * i;
-      if (v < nvec) part = fmaf(dot_vec<QT>(w[i], load_x<QT>(hp + v * Vec<QT>::kW)), sc[i], part);
+      for (int i = 0; i < VPL; ++i) {
+        const int v = lane + 32 * i;
+        if (v < nvec) part = fmaf(dot_vec<QT>(w[i], staged_x<QT>(hs, nvec, v)), sc[i], part);
+      }
+      part = warp_sum(part);
+      if (lane == 0) d.part[(size_t)d.asg[c0 + t] * d.H + c] = part;
     }
-    part = warp_sum(part);
-    if (lane == 0) d.part[(size_t)pos * d.H + c] = part;
   }
 }
 
@@ -169,6 +216,16 @@ __global__ void k_combine(Dev d, int T, float* __restrict__ y) {
   y[i] = acc;
 }
 
+// Kernels of calls with several waves run beside the side stream's materialiser, which asks for
+// the largest shared-memory carveout (an SM holds blocks of one carveout at a time): they ask
+// for the same, once per kernel.
+template <class K>
+cudaError_t same_carveout(K kern) {
+  static cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                              cudaSharedmemCarveoutMaxShared);
+  return e;
+}
+
 // smallest instantiated vectors-per-lane count covering `nvec` vectors
 int pick_vpl(int nvec) {
   const int need = (nvec + 31) / 32;
@@ -180,18 +237,24 @@ int pick_vpl(int nvec) {
   return 8;
 }
 
+template <int QT, int VPL>
+cudaError_t launch_gateup_v(const Dev& d, int layer, int wave, int width, const float* x, cudaStream_t s) {
+  const cudaError_t e = same_carveout(k_gateup<QT, VPL>);
+  if (e != cudaSuccess) return e;
+  k_gateup<QT, VPL><<<dim3((d.I + 7) / 8, width), 256, 0, s>>>(d, layer, wave, x);
+  return cudaGetLastError();
+}
+
 template <int QT>
 cudaError_t gateup_q(const Dev& d, int layer, int wave, int width, const float* x, cudaStream_t s) {
-  dim3 grid((d.I + 7) / 8, width);
   switch (pick_vpl(d.lay.qrow_gu / 16)) {
-    case 1: k_gateup<QT, 1><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
-    case 2: k_gateup<QT, 2><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
-    case 3: k_gateup<QT, 3><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
-    case 4: k_gateup<QT, 4><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
-    case 6: k_gateup<QT, 6><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
-    default: k_gateup<QT, 8><<<grid, 256, 0, s>>>(d, layer, wave, x); break;
+    case 1: return launch_gateup_v<QT, 1>(d, layer, wave, width, x, s);
+    case 2: return launch_gateup_v<QT, 2>(d, layer, wave, width, x, s);
+    case 3: return launch_gateup_v<QT, 3>(d, layer, wave, width, x, s);
+    case 4: return launch_gateup_v<QT, 4>(d, layer, wave, width, x, s);
+    case 6: return launch_gateup_v<QT, 6>(d, layer, wave, width, x, s);
+    default: return launch_gateup_v<QT, 8>(d, layer, wave, width, x, s);
   }
-  return cudaGetLastError();
 }
 
 template <int QT>
@@ -208,18 +271,28 @@ cudaError_t down_single_q(const Dev& d, int layer, float* y, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+template <int QT, int VPL>
+cudaError_t launch_down_partial_v(const Dev& d, int layer, int wave, int width, cudaStream_t s) {
+  constexpr int RB = rows_per_block<QT, VPL>();
+  const size_t smem = (size_t)chunk_tokens(d.I) * d.I * sizeof(float);
+  cudaError_t e =
+      cudaFuncSetAttribute(k_down_partial<QT, VPL>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess) e = same_carveout(k_down_partial<QT, VPL>);
+  if (e != cudaSuccess) return e;
+  k_down_partial<QT, VPL><<<dim3((d.H + RB - 1) / RB, width), RB * 32, smem, s>>>(d, layer, wave);
+  return cudaGetLastError();
+}
+
 template <int QT>
 cudaError_t down_partial_q(const Dev& d, int layer, int wave, int width, cudaStream_t s) {
-  dim3 grid((d.H + 7) / 8, width);
   switch (pick_vpl(d.lay.qrow_d / 16)) {
-    case 1: k_down_partial<QT, 1><<<grid, 256, 0, s>>>(d, layer, wave); break;
-    case 2: k_down_partial<QT, 2><<<grid, 256, 0, s>>>(d, layer, wave); break;
-    case 3: k_down_partial<QT, 3><<<grid, 256, 0, s>>>(d, layer, wave); break;
-    case 4: k_down_partial<QT, 4><<<grid, 256, 0, s>>>(d, layer, wave); break;
-    case 6: k_down_partial<QT, 6><<<grid, 256, 0, s>>>(d, layer, wave); break;
-    default: k_down_partial<QT, 8><<<grid, 256, 0, s>>>(d, layer, wave); break;
+    case 1: return launch_down_partial_v<QT, 1>(d, layer, wave, width, s);
+    case 2: return launch_down_partial_v<QT, 2>(d, layer, wave, width, s);
+    case 3: return launch_down_partial_v<QT, 3>(d, layer, wave, width, s);
+    case 4: return launch_down_partial_v<QT, 4>(d, layer, wave, width, s);
+    case 6: return launch_down_partial_v<QT, 6>(d, layer, wave, width, s);
+    default: return launch_down_partial_v<QT, 8>(d, layer, wave, width, s);
   }
-  return cudaGetLastError();
 }
 
 }  // namespace
@@ -238,6 +311,7 @@ cudaError_t launch_down_partial(const Dev& d, int layer, int wave, int width, cu
 
 cudaError_t launch_combine(const Dev& d, int T, float* y, cudaStream_t s) {
   const size_t n = (size_t)T * d.H;
+  same_carveout(k_combine);
   k_combine<<<(unsigned)((n + 255) / 256), 256, 0, s>>>(d, T, y);
   return cudaGetLastError();
 }

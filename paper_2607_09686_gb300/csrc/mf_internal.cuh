@@ -37,6 +37,7 @@ struct Dev {
   // model
   int L, H, E, k, I, qtype;
   int S_alloc, S_active, T_max;
+  int order;  // access order of calls with T > 1 (MF_ORDER_*)
   Layout lay;
   // memory
   const uint8_t* pack;  // pinned host pack [L][E] slots, device-addressable
@@ -176,9 +177,10 @@ size_t router_part_pairs(int T_max, int E, int H);
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
                           cudaStream_t s, float* x_copy = nullptr);
 cudaError_t launch_resolve(const Dev& d, int layer, int T, cudaStream_t s);
-// dst_stage null: each miss into its slot; else miss m of the wave to dst_stage + m * stride
+// dst_stage null: each miss into its slot; else miss m of the wave to dst_stage + m * stride.
+// spread: one small block per SM (beside the persistent GEMM kernels), else a few large blocks
 cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s,
-                               uint8_t* dst_stage = nullptr);
+                               uint8_t* dst_stage = nullptr, bool spread = false);
 // the wave's staged payloads into their slots
 cudaError_t launch_stage_commit(const Dev& d, int layer, int wave, const uint8_t* stage, cudaStream_t s);
 cudaError_t launch_gateup(const Dev& d, int layer, int wave, int wave_width, const float* x, cudaStream_t s);

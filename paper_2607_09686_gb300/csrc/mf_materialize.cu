@@ -4,9 +4,14 @@
 // The misses are decided on the device (slot resolve), so the copy is driven by the GPU
 // itself: SMs load 16-byte vectors straight from the pinned, device-mapped pack over the
 // CPU-GPU link and store them into the slot, with no host round trip.  Launched on the
-// context's side stream: one small block per SM (two warps, 8 KB of loads in flight each: the
-// link saturates at a fraction of that) strides over each missed payload of the wave in turn;
-// with no miss every block returns at once.  Both kernels here ask
+// context's side stream, blocks stride over each missed payload of the wave in turn (with no
+// miss every block returns at once), 8 16-byte loads in flight per thread, 1.2 MB in all: the
+// link saturates at about that.  Where they go matters for the kernel computing beside them:
+// an SM with long-latency host loads outstanding serves its other blocks' memory requests
+// slowly.  So the dequantising GEMV kernels (many small blocks, scheduled as SMs free up) get
+// the copy concentrated on one SM in eight (large blocks), while the persistent GEMM kernels
+// (one block per SM with a fixed share of the work) get it spread thin over every SM.  Both
+// kernels here ask
 // for the largest shared-memory carveout although they use none: an SM runs blocks of one
 // carveout at a time, so only then can they share SMs with a running expert-FFN kernel (which
 // needs most of the shared memory) instead of holding those SMs until they finish.
@@ -20,11 +25,12 @@ namespace mf {
 namespace {
 
 constexpr int kUnroll = 8;
-constexpr int kMatThreads = 64;
+constexpr int kMatThreadsSpread = 64;  // one block per SM
+constexpr int kMatThreadsDense = 512;  // one block per 8 SMs
 
 // dst_stage: null to write each miss into its slot, else miss m of the wave goes to
 // dst_stage + m * stride
-__global__ void __launch_bounds__(kMatThreads) k_materialize(Dev d, int layer, int wave, uint8_t* dst_stage) {
+__global__ void __launch_bounds__(kMatThreadsDense) k_materialize(Dev d, int layer, int wave, uint8_t* dst_stage) {
   const int n_miss = d.info[2 + wave];
   const size_t nvec = d.lay.stride / 16;  // 16-byte vectors per payload
   const size_t step = (size_t)gridDim.x * blockDim.x * kUnroll;
@@ -99,11 +105,15 @@ cudaError_t max_shared_carveout() {
   return e;
 }
 
-cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s, uint8_t* dst_stage) {
+cudaError_t launch_materialize(const Dev& d, int layer, int wave, int max_miss, cudaStream_t s, uint8_t* dst_stage,
+                               bool spread) {
   if (max_miss <= 0) return cudaSuccess;
   cudaError_t e = max_shared_carveout();
   if (e != cudaSuccess) return e;
-  k_materialize<<<n_sm(), kMatThreads, 0, s>>>(d, layer, wave, dst_stage);
+  if (spread)
+    k_materialize<<<n_sm(), kMatThreadsSpread, 0, s>>>(d, layer, wave, dst_stage);
+  else
+    k_materialize<<<(n_sm() + 7) / 8, kMatThreadsDense, 0, s>>>(d, layer, wave, dst_stage);
   return cudaGetLastError();
 }
 

@@ -4,7 +4,8 @@
 //
 // One block of 1024 threads per call.  Steps:
 //  1. the distinct experts of the call's T*k routes, in (token, rank) first-occurrence
-//     order, and for each the list of assignments t*k+j it serves;
+//     order (or, with MF_ORDER_RESIDENT_FIRST, the resident ones first), and for each the list
+//     of assignments t*k+j it serves;
 //  2. least-recently-used replacement over those accesses in waves of S (lru_block);
 //  3. counters (accesses, hits, misses, evictions, bytes = misses * payload) and the
 //     access record of the call.
@@ -111,6 +112,22 @@ __global__ void __launch_bounds__(kThreadsRes, 1) k_resolve(Dev d, int layer, in
   }
   __syncthreads();
   const int U = s_U;
+  if (d.order == MF_ORDER_RESIDENT_FIRST) {  // stable: resident experts first, then the others
+    int* tmp = s_uslot;                      // reused (written by the LRU below)
+    for (int u = tid; u < U; u += nt) tmp[u] = s_uniq[u];
+    __syncthreads();
+    int n_res = 0;
+    for (int v = 0; v < U; ++v) n_res += s_slot_of[tmp[v]] >= 0;
+    for (int u = tid; u < U; u += nt) {
+      const int e = tmp[u];
+      const bool res = s_slot_of[e] >= 0;
+      int r = res ? 0 : n_res;
+      for (int v = 0; v < u; ++v) r += (s_slot_of[tmp[v]] >= 0) == res;
+      s_uniq[r] = e;
+      uidx[e] = r;
+    }
+    __syncthreads();
+  }
   int* ucnt = firstpos;  // reused: routes of the u-th distinct expert
   for (int u = tid; u < U; u += nt) ucnt[u] = cnt[s_uniq[u]];
   __syncthreads();

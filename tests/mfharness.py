@@ -124,8 +124,8 @@ class Ctx:
         return out
 
 
-def oracle_trace(lru: oracle.LRU, idx: np.ndarray):
-    u, sl, hit = lru.step(idx)
+def oracle_trace(lru: oracle.LRU, idx: np.ndarray, order: int = 0):
+    u, sl, hit = lru.step(idx, order)
     return list(map(int, u)), list(map(int, sl)), list(map(bool, hit))
 
 

@@ -96,11 +96,12 @@ def test_q4_0_decode_full_width(kernels, monkeypatch):
     _decode_run(shape, 19, 24, seed=2, route=synth.configs.ZIPF12, sample_y=12)
 
 
-def _batch_run(shape, slots, T, n_steps, seed, zipf_s=1.0, layers=None, sample_tokens=None):
+def _batch_run(shape, slots, T, n_steps, seed, zipf_s=1.0, layers=None, sample_tokens=None, order=0):
     layers = list(range(shape.n_layers)) if layers is None else layers
     ctx = Ctx(shape, slots, max_tokens=T)
     pays = Payloads(shape)
     try:
+        ctx.mf.mf_access_order(ctx.h, order)
         H, E, k = shape.hidden, shape.n_experts, shape.top_k
         lru = {l: oracle.LRU(E, slots, synth.payload_bytes(H, shape.inter, shape.qtype)) for l in layers}
         routes = {l: np.stack([synth.routes(seed, l, s, E, k, n_steps, zipf_s, 0.0) for s in range(T)], 1)
@@ -114,17 +115,20 @@ def _batch_run(shape, slots, T, n_steps, seed, zipf_s=1.0, layers=None, sample_t
                     _, oidx, og = oracle.router(x[t], ctx.wr_host[l], b[t], k)
                     assert np.array_equal(idx[t], oidx)
                     assert np.abs(w[t] - og).max() <= G_ATOL
-                assert tr == oracle_trace(lru[l], idx), (l, step)
+                assert tr == oracle_trace(lru[l], idx, order), (l, step)
                 toks = range(T) if sample_tokens is None else sorted(
                     set(np.random.default_rng(step * 131 + l).integers(0, T, sample_tokens).tolist()))
                 for t in toks:
                     yo, _, _ = oracle.layer(pays.for_layer(l, idx[t]), shape.qtype, H, shape.inter, k,
                                             ctx.wr_host[l], b[t:t + 1], x[t:t + 1])
                     assert_outputs_close(y[t:t + 1], yo, f"layer {l} step {step} token {t}")
+        out = []
         for l in layers:
             st, ost = ctx.mf.mf_stats(ctx.h, l), lru[l].stats()
             assert (st["hits"], st["misses"], st["evictions"], st["bytes_materialized"]) == \
                 (ost["hits"], ost["misses"], ost["evictions"], ost["bytes"])
+            out.append(st)
+        return out
     finally:
         ctx.close()
 
@@ -133,6 +137,17 @@ def _batch_run(shape, slots, T, n_steps, seed, zipf_s=1.0, layers=None, sample_t
 def test_batched_steps_in_waves(qtype):
     """16 tokens x top-3 over 12 experts with 4 slots: up to 3 waves per step."""
     _batch_run(Shape(2, 96, 12, 3, 160, qtype, model_seed=9), 4, 16, 6, seed=1, zipf_s=0.5)
+
+
+@pytest.mark.parametrize("qtype", [synth.Q8_0, synth.Q4_0])
+def test_batched_steps_resident_first(qtype):
+    """The same batched steps with the resident-first access order: routes, traces (access order,
+    slots, hits), counters and outputs against the oracle in that order; never fewer hits than
+    the first-occurrence order on these steps."""
+    shape = Shape(2, 96, 12, 3, 160, qtype, model_seed=9)
+    rf = _batch_run(shape, 4, 16, 6, seed=1, zipf_s=0.5, order=1)
+    fo = _batch_run(shape, 4, 16, 6, seed=1, zipf_s=0.5, order=0)
+    assert sum(s["hits"] for s in rf) >= sum(s["hits"] for s in fo)
 
 
 def test_max_experts_and_many_waves():
@@ -262,5 +277,11 @@ def test_argument_and_state_errors():
         torch.cuda.synchronize()
         with pytest.raises(mf.MFError):
             mf.mf_reset(h, 1)  # fewer slots than top-k
+        for bad in (-1, 2):
+            with pytest.raises(mf.MFError) as e:
+                mf.mf_access_order(h, bad)
+            assert e.value.status == mf.MF_E_INVAL
+        mf.mf_access_order(h, mf.MF_ORDER_RESIDENT_FIRST)
+        mf.mf_access_order(h, mf.MF_ORDER_FIRST_OCCURRENCE)
     finally:
         mf.mf_destroy(h)

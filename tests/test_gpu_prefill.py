@@ -102,6 +102,34 @@ def test_gemm_l4e64_shape(qtype):
         ctx.close()
 
 
+def test_gemm_resident_first_order():
+    """The GEMM path with the resident-first order: 2 calls of 320 tokens on one layer (the second
+    with most experts resident), every output, index, access record and counter against the
+    oracle in that order."""
+    cfg = synth.CONFIGS["l4e64"]
+    shape = Shape(1, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, synth.Q4_0, model_seed=4)
+    ctx = Ctx(shape, slots=22, max_tokens=320)
+    try:
+        ctx.mf.mf_access_order(ctx.h, 1)
+        pays = Payloads(shape)
+        lru = oracle.LRU(shape.n_experts, 22, synth.payload_bytes(shape.hidden, shape.inter, shape.qtype))
+        for call in range(2):
+            r = synth.routes(8, 0, call, shape.n_experts, shape.top_k, 320, 1.1, 0.0)
+            x = synth.activations(8, 0, call, 0, 320, shape.hidden)
+            bias = synth.plant_bias(r, shape.n_experts)
+            y, idx, w, tr = ctx.forward(0, x, bias, 320, trace=True)
+            yo, oidx, og = oracle.layer(pays.for_layer(0, np.unique(idx)), shape.qtype, shape.hidden, shape.inter,
+                                        shape.top_k, ctx.wr_host[0], bias, x)
+            assert np.array_equal(idx, oidx) and np.abs(w - og).max() <= G_ATOL
+            assert tr == oracle_trace(lru, idx, 1), call
+            assert_outputs_close(y, yo, f"call {call}")
+        st, ost = ctx.mf.mf_stats(ctx.h, 0), lru.stats()
+        assert (st["hits"], st["misses"], st["evictions"]) == (ost["hits"], ost["misses"], ost["evictions"])
+        assert ctx.mf.mf_check(ctx.h) == 0
+    finally:
+        ctx.close()
+
+
 def test_gemm_matches_gemv_path():
     """Same inputs through the GEMM path and the GEMV path: same routes, access sequence and
     counters; outputs agree within the oracle tolerance of each other."""

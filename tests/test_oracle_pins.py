@@ -289,6 +289,46 @@ def test_lru_uniform_hit_rate_closed_form():
     assert abs(rate - expect) < 0.012  # ~4 standard deviations of 22400 Bernoulli draws
 
 
+def test_lru_resident_first_worked_example():
+    """Two slots holding experts 0 and 1 (0 least recent); a step of two tokens routed [2, 3] then
+    [0, 1].  First-occurrence order: 2 and 3 miss and evict 0 and 1, which then miss too (4
+    misses).  Resident first: 0 and 1 hit, then 2 and 3 miss into their slots (2 misses)."""
+    step = np.array([[2, 3], [0, 1]], np.int32)
+    first, res = oracle.LRU(4, 2, 1), oracle.LRU(4, 2, 1)
+    for c in (first, res):
+        c.step(np.array([[0, 1]], np.int32))  # 0 then 1: 0 is least recent
+    u, sl, h = first.step(step, order=0)
+    assert (list(u), list(sl), list(h)) == ([2, 3, 0, 1], [0, 1, 0, 1], [False] * 4)
+    u, sl, h = res.step(step, order=1)
+    assert (list(u), list(sl), list(h)) == ([0, 1, 2, 3], [0, 1, 0, 1], [True, True, False, False])
+    assert (first.stats()["misses"], res.stats()["misses"]) == (2 + 4, 2 + 2)
+
+
+@pytest.mark.parametrize("S,T,s", [(4, 8, 0.8), (9, 16, 1.1), (19, 64, 1.0), (6, 2, 0.0)])
+def test_lru_resident_first_against_textbook(S, T, s):
+    """Resident-first steps on the textbook cache: the access list is the step's distinct
+    experts resident at its start (first-occurrence order), then the rest; every one of the
+    former hits; decisions and slots as the textbook LRU gives them for that sequence; and a
+    step never has fewer hits than the residents it needs."""
+    E, k = 32, 4
+    r = synth.routes(11, 0, 0, E, k, 40 * T, s, 0.3)
+    orc, ref = oracle.LRU(E, S, 1), TextbookLRU(S)
+    for step in _steps_from_routes(r, T):
+        seen = []
+        for e in step.reshape(-1):
+            if int(e) not in seen:
+                seen.append(int(e))
+        resident = [e for e in seen if e in ref.d] if T > 1 else []
+        order = resident + [e for e in seen if e not in resident] if T > 1 else seen
+        uniq, slot, hit = orc.step(step, order=1)
+        assert list(uniq) == order
+        for u, e in enumerate(order):
+            h, sl = ref.access(e)
+            assert (bool(hit[u]), int(slot[u])) == (h, sl)
+        assert all(hit[:len(resident)])
+        assert orc.occupancy() <= S
+
+
 # ---------------------------------------------------------------- static budget check
 def test_plan_closed_form_l30e128():
     for line in golden_lines("plan_l30e128b64.txt"):
