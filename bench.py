@@ -328,8 +328,12 @@ def run_mawforge(args):
                                                             args.steps, rf_bytes, hbm)
     if not args.no_prefill:
         line["prefill"] = prefill_measurement(torch, mf, synth, device)
+    if not args.no_batch64:
+        line["batch64"] = batch64_measurement(torch, mf, synth, device)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
+        runs = [cpu_baseline(args.cpu_tokens) for _ in range(args.cpu_passes)]
+        line["cpu_baseline"] = dict(runs[0], value=round(statistics.mean(r["value"] for r in runs), 4),
+                                    sample=runs[0]["sample"] + f", {args.cpu_passes} passes from a cold cache")
     if rank == 0:
         print(json.dumps(line))
     if ws > 1:
@@ -473,6 +477,58 @@ def prefill_measurement(torch, mf, synth, device, calls: int = 4, cache_pct: flo
                          "flops_per_call": {"useful": useful, "issued": issued}}}
 
 
+def batch64_measurement(torch, mf, synth, device, steps: int = 8, warm: int = 2, cache_pct: float = 15.0) -> dict:
+    """64 concurrent decode streams on one layer of the 30-layer workload (hidden 2816, 128
+    experts, top-8, inter 1408, Q8_0, Zipf 1.0 per stream) at 15 % cache: one call of T = 64 per
+    step (~107 distinct experts against 19 slots: 6 waves, their misses over the host link), for
+    both access orders.  CUDA events around `steps` calls after `warm` calls."""
+    cfg = synth.CONFIGS["l30e128b64"]
+    H, E, k, I, q, B = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype, cfg.batch
+    model = mf.Model(1, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(cache_pct, 1 << 62, 0, 0, B, 0))
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    out = {"workload": f"l30e128b64 layer 0: {B} decode streams per call, hidden {H}, {E} experts, top-{k}, "
+                       f"inter {I}, Q8_0, Zipf {cfg.route_classes[0].zipf_s:g} per stream, cache {cache_pct:g}% "
+                       f"({plan.slots_per_layer} slots)"}
+    try:
+        buf = np.empty(plan.payload_bytes, np.uint8)
+        for e in range(E):
+            synth.payload(cfg.model_seed, 0, e, H, I, q, out=buf)
+            mf.mf_pack_put(ctx, 0, e, buf)
+        n = warm + steps
+        klass = cfg.route_classes[0]
+        routes = np.stack([synth.routes(0, 0, st, E, k, n, klass.zipf_s, klass.reuse) for st in range(B)], 1)
+        wr = torch.from_numpy(synth.router_weights(cfg.model_seed, 0, E, H)).to(device)
+        xs = [torch.from_numpy(np.concatenate([synth.activations(0, 0, st, i, 1, H) for st in range(B)])).to(device)
+              for i in range(n)]
+        bs = [torch.from_numpy(synth.plant_bias(routes[i], E)).to(device) for i in range(n)]
+        y = torch.empty(B, H, device=device)
+        for name, order in (("first_occurrence", mf.MF_ORDER_FIRST_OCCURRENCE),
+                            ("resident_first", mf.MF_ORDER_RESIDENT_FIRST)):
+            mf.mf_reset(ctx)
+            mf.mf_access_order(ctx, order)
+            for i in range(warm):
+                mf.mf_moe_forward(ctx, 0, xs[i], wr, bs[i], B, y)
+            torch.cuda.synchronize()
+            mf.mf_stats(ctx, 0, reset=True)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            for i in range(warm, n):
+                mf.mf_moe_forward(ctx, 0, xs[i], wr, bs[i], B, y)
+            b.record()
+            b.synchronize()
+            ms = a.elapsed_time(b) / steps
+            st = mf.mf_stats(ctx, 0)
+            out[name] = {"tokens_per_s": round(B / (ms * 1e-3), 1), "ms_per_step": round(ms, 4),
+                         "hit_rate": round(st["hits"] / st["accesses"], 4),
+                         "materialized_mb_per_step": round(st["bytes_materialized"] / steps / 1e6, 2),
+                         "link_gbs": round(st["bytes_materialized"] / steps / (ms * 1e-3) / 1e9, 1)}
+        assert mf.mf_check(ctx) == 0
+    finally:
+        mf.mf_destroy(ctx)
+    return out
+
+
 def _bf16_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -505,7 +561,8 @@ def cpu_baseline(n_tokens: int) -> dict:
     dt = time.perf_counter() - t0
     cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     return {"value": round(n_tokens / dt, 4), "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"first {n_tokens} tokens of the same sequence, all {L} layers (router + LRU + fp64 layer)"}
+            "sample": f"first {n_tokens} tokens of the same sequence (256 = the whole step), all {L} layers "
+                      "(router + LRU + fp64 layer)"}
 
 
 def run_reference(args):
@@ -537,10 +594,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--cache-pct", type=float, default=35.0)
     ap.add_argument("--impl", default="mawforge", choices=["mawforge", "reference"])
-    ap.add_argument("--cpu-tokens", type=int, default=16)
+    ap.add_argument("--cpu-tokens", type=int, default=256, help="tokens of the sequence the CPU oracle runs per pass")
+    ap.add_argument("--cpu-passes", type=int, default=3, help="passes of the CPU baseline leg (~3 s each)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prefill", action="store_true", help="skip the 4096-token prefill measurement")
     ap.add_argument("--no-resident", action="store_true", help="skip the all-resident FFN measurement")
+    ap.add_argument("--no-batch64", action="store_true", help="skip the 64-stream batched decode measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle
