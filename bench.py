@@ -109,6 +109,22 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def max_over_ranks(torch, v: float, device) -> float:
+    """The largest of the ranks' values (a job ends with its slowest rank); v itself on one rank."""
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return v
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank: float, ms_max: float, ws: int) -> float:
+    """Whole-job throughput: every rank's units (weak scaling: the same on each) over the slowest
+    rank's time."""
+    return units_per_rank * ws / (ms_max * 1e-3)
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -209,11 +225,7 @@ def run_mawforge(args):
     step_ms = [a.elapsed_time(b) for a, b in evs]
     ms = sum(step_ms) / len(step_ms)
     ms_instrumented = sum(a.elapsed_time(b) for a, b in evk) / len(evk)
-    if ws > 1:
-        t = torch.tensor([ms], device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        torch.distributed.barrier()
-        ms = float(t.item())
+    ms = max_over_ranks(torch, ms, device)
     st = mf.mf_stats(ctx, -1)  # every step starts cold (mf_reset), so these are one step's counters
     mf.mf_timing(ctx, [])
 
@@ -270,7 +282,8 @@ def run_mawforge(args):
     gemv_ms = ms_ff + ms_gu + ms_dn
     gemv_gbs = (gu_bytes + dn_bytes) * (n_ff + n_gu) / (gemv_ms * 1e-3) / 1e9
     tokens = N_TOKENS * args.steps * ws
-    value = N_TOKENS / (ms * 1e-3) * ws
+    value = job_rate(N_TOKENS, ms, ws)
+    e2e_ms_max = max_over_ranks(torch, statistics.mean(e2e_ms), device)
     clocks = clk.summary()
     kernels = {name: {"ms_total": round(v[0], 4), "launches": v[1],
                       "us_per_launch": round(1e3 * v[0] / v[1], 3) if v[1] else None} for name, v in kt.items()}
@@ -314,7 +327,7 @@ def run_mawforge(args):
                  "note": "one-token calls materialise inside the fused FFN launch; the lower bound divides "
                          "the materialised bytes by all of that kernel's time"},
         "clocks": clocks,
-        "e2e": {"value": round(N_TOKENS / (statistics.mean(e2e_ms) * 1e-3) * ws, 2), "unit": "tokens/s",
+        "e2e": {"value": round(job_rate(N_TOKENS, e2e_ms_max, ws), 2), "unit": "tokens/s",
                 "h2d_bytes_per_step": N_TOKENS * L * (H + E) * 4, "d2h_bytes_per_step": N_TOKENS * L * H * 4},
         "gpu_launches": None,
         "wall_s": round(wall, 3),
@@ -323,12 +336,12 @@ def run_mawforge(args):
     # the same calls), one router per call and one reset per step
     line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps * (N_TOKENS * L + 1)
     mf.mf_destroy(ctx)
-    if n_ff and not args.no_resident:
+    if n_ff and not args.no_resident and rank == 0:
         line["roofline"]["resident"] = resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush,
                                                             args.steps, rf_bytes, hbm)
-    if not args.no_prefill:
+    if not args.no_prefill and rank == 0:
         line["prefill"] = prefill_measurement(torch, mf, synth, device)
-    if not args.no_batch64:
+    if not args.no_batch64 and rank == 0:
         line["batch64"] = batch64_measurement(torch, mf, synth, device)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         runs = [cpu_baseline(args.cpu_tokens) for _ in range(args.cpu_passes)]
