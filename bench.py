@@ -180,7 +180,7 @@ def run_mawforge(args):
     # timed steps replay a graph without instrumentation; the per-kernel breakdown comes from the
     # same calls captured a second time with the library's CUDA-event records around each launch
     # (graph nodes, so they time the launches of those replays), replayed right after.
-    timed = ["materialize", "ffn_fused", "gateup_swiglu", "down_combine"]
+    timed = ["router", "resolve", "materialize", "ffn_fused", "gateup_swiglu", "down_combine"]
     graph, graph_k = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
     with torch.cuda.stream(stream):
         step_calls()  # untimed eager pass: warms the pool
@@ -333,8 +333,8 @@ def run_mawforge(args):
         "wall_s": round(wall, 3),
     }
     # every kernel of the timed replays: the timed classes (counted in the instrumented replays of
-    # the same calls), one router per call and one reset per step
-    line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps * (N_TOKENS * L + 1)
+    # the same calls) and one reset per step
+    line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps
     mf.mf_destroy(ctx)
     if n_ff and not args.no_resident and rank == 0:
         line["roofline"]["resident"] = resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush,

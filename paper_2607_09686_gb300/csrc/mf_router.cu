@@ -209,6 +209,9 @@ __global__ void __launch_bounds__(kThreadsR)
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 
   // rank by counting: position of expert e = experts with a larger logit, or equal and lower id
+  // (s_sel starts as 0..k-1: a valid choice even where the logits are not ordered, e.g. NaN)
+  if (tid < k) s_sel[tid] = tid;
+  __syncthreads();
   for (int e = tid; e < E; e += kThreadsR) {
     const float z = s_z[e];
     int r = 0;
@@ -414,6 +417,8 @@ __global__ void __launch_bounds__(kTokW * 32)
     if (bias) v = __fadd_rn(v, bias[(size_t)t * E + e]);
     z[e] = v;
   }
+  __syncwarp();
+  if (lane < k) s_sel[warp][lane] = lane;  // valid even where the logits are not ordered (NaN)
   __syncwarp();
   for (int e = lane; e < E; e += 32) {  // rank by counting, ties to the lower id
     const float v = z[e];
