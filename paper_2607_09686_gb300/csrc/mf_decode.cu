@@ -454,13 +454,14 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     const size_t doff = (size_t)r0 * d.lay.rs_d;
     // the resident experts' down records go after the first two gate/up items
     const int first = min(nres, min(2, NA));
+    const uint64_t pol = l2_evict_first();  // read once per call: keep L2 for what is reused
     bool d_issued = false;
     auto issue_down_hits = [&]() {
       if (lane == 0)
         for (int j = 0; j < mine_d; ++j)
           if (!s_miss[j]) {
             mbar_arrive_tx(&full_d[j], dbytes);
-            bulk_g2s(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, dbytes, &full_d[j]);
+            bulk_g2s_hint(dbuf + (size_t)j * f.dn_bytes, s_dn[j] + doff, dbytes, &full_d[j], pol);
           }
       d_issued = true;
     };
@@ -471,7 +472,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
         const int item = s_gord[t], u = item / nrb, rb = item % nrb;
         uint64_t* bar = &sm.full[ring.s];
         mbar_arrive_tx(bar, bytes);
-        bulk_g2s(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar);
+        bulk_g2s_hint(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar, pol);
         ring.next(NA);
       }
       if (ok && !d_issued) issue_down_hits();

@@ -65,10 +65,11 @@ __device__ __forceinline__ void pair_add(float& s, float& c, float s2, float c2)
 // The first chunk of logit_part's W loads, issued before x is in shared memory.
 __device__ __forceinline__ void w_preload(const float* __restrict__ w, int n4, int first, int step, float4* a) {
   const float4* w4 = reinterpret_cast<const float4*>(w);
+  const uint64_t pol = l2_evict_last();  // W_r is read again by the layer's next call
 #pragma unroll
   for (int u = 0; u < kChunk; ++u) {
     const int q = first + u * step;
-    if (q < n4) a[u] = __ldg(w4 + q);
+    if (q < n4) a[u] = ld_hint(w4 + q, pol);
   }
 }
 
@@ -87,7 +88,7 @@ __device__ __forceinline__ void logit_part(const float* __restrict__ w, const fl
     for (int u = 0; u < kChunk; ++u) {  // all loads of the chunk first
       const int q = q0 + u * step;
       if (q < n4) {
-        a[u] = q0 == first ? pre[u] : __ldg(w4 + q);
+        a[u] = q0 == first ? pre[u] : ld_hint(w4 + q, l2_evict_last());
         b[u] = x4[q];
       }
     }
