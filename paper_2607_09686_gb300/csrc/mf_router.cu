@@ -210,27 +210,29 @@ __global__ void __launch_bounds__(kThreadsR)
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 
   // rank by counting: position of expert e = experts with a larger logit, or equal and lower id
-  // (s_sel starts as 0..k-1: a valid choice even where the logits are not ordered, e.g. NaN)
+  // (s_sel starts as 0..k-1: a valid choice even where the logits are not ordered, e.g. NaN).
+  // tpe consecutive lanes share an expert, each counting over every tpe-th other expert.
   if (tid < k) s_sel[tid] = tid;
   __syncthreads();
-  for (int e = tid; e < E; e += kThreadsR) {
-    const float z = s_z[e];
-    int r = 0;
-    for (int e4 = 0; e4 < E / 4; ++e4) {  // s_z is 16-byte aligned; E % 4 tail below
-      const float4 z4 = reinterpret_cast<const float4*>(s_z)[e4];
-      const int b = 4 * e4;
-      r += (z4.x > z) || (z4.x == z && b < e);
-      r += (z4.y > z) || (z4.y == z && b + 1 < e);
-      r += (z4.z > z) || (z4.z == z && b + 2 < e);
-      r += (z4.w > z) || (z4.w == z && b + 3 < e);
-    }
-    for (int e2 = E & ~3; e2 < E; ++e2) {
-      const float z2 = s_z[e2];
-      r += (z2 > z) || (z2 == z && e2 < e);
-    }
-    if (r < k) {
-      s_sel[r] = e;
-      s_zsel[r] = z;
+  {
+    int tpe = 1;
+    while (tpe < 32 && tpe * 2 * E <= kThreadsR) tpe *= 2;
+    const int per_pass = kThreadsR / tpe, part = tid % tpe;
+    for (int e0 = 0; e0 < E; e0 += per_pass) {  // block-uniform
+      const int e = e0 + tid / tpe;
+      const bool valid = e < E;
+      const float z = valid ? s_z[e] : 0.f;
+      int r = 0;
+      if (valid)
+        for (int e2 = part; e2 < E; e2 += tpe) {
+          const float z2 = s_z[e2];
+          r += (z2 > z) || (z2 == z && e2 < e);
+        }
+      for (int off = tpe >> 1; off > 0; off >>= 1) r += __shfl_xor_sync(0xffffffffu, r, off);
+      if (valid && part == 0 && r < k) {
+        s_sel[r] = e;
+        s_zsel[r] = z;
+      }
     }
   }
   __syncthreads();
