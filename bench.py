@@ -336,6 +336,12 @@ def run_mawforge(args):
     # the same calls) and one reset per step
     line["gpu_launches"] = int(sum(v[1] for v in kt.values())) + args.steps
     mf.mf_destroy(ctx)
+    h2d = h2d_bandwidth(torch, device, stream)
+    link_ms = st["bytes_materialized"] / (h2d * 1e9) * 1e3
+    line["copy"].update({"h2d_gbs_measured": round(h2d, 1),
+                         "link_ms_per_step_at_h2d": round(link_ms, 3),
+                         "link_share_of_step": round(link_ms / ms, 4),
+                         "h2d_how": "pinned host -> device cudaMemcpyAsync of 1 GiB, best of 3, this run"})
     if n_ff and not args.no_resident and rank == 0:
         line["roofline"]["resident"] = resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush,
                                                             args.steps, rf_bytes, hbm)
@@ -403,6 +409,24 @@ def resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, s
             "misses_in_timed_replays": st["misses"],
             "how": "same calls, 100 % cache warmed by two passes (every launch all-resident), L2 flushed per replay",
             "read_floor": read_floor(torch, device, stream, flush, bytes_per_launch, hbm)}
+
+
+def h2d_bandwidth(torch, device, stream, nbytes: int = 1 << 30, reps: int = 3) -> float:
+    """GB/s of one pinned host -> device copy engine transfer (the CPU-GPU link's rate for a
+    plain copy), best of `reps`."""
+    src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    dst = torch.empty(nbytes, dtype=torch.uint8, device=device)
+    best = 0.0
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            dst.copy_(src, non_blocking=True)
+            b.record(stream)
+            b.synchronize()
+            best = max(best, nbytes / (a.elapsed_time(b) * 1e-3) / 1e9)
+    del src, dst
+    return best
 
 
 def read_floor(torch, device, stream, flush, nbytes, hbm, reps: int = 20) -> dict:
