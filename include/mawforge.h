@@ -220,10 +220,11 @@ int mf_check(mf_ctx_t* ctx);
  *   experts  device, 16-byte aligned: top_k expert slots back to back, slot j = expert j, each
  *            `stride` bytes in this layout (Q = bytes of codes per row: hidden (Q8_0) or
  *            hidden/2 (Q4_0) for gate/up rows, inter or inter/2 for down rows; nb = weights/32):
- *              rs_gu = round16(2*Q_gu + 4*nb_gu), rs_d = round16(Q_d + 2*nb_d),
+ *              rs_gu = round16(2*Q_gu + round16(2*nb_gu) + 2*nb_gu), rs_d = round16(Q_d + 2*nb_d),
  *              d_off = round256(inter * rs_gu), stride = round256(d_off + hidden * rs_d);
  *              gate/up record r at r*rs_gu: [gate codes row r][up codes row r]
- *                [gate scales row r (nb_gu binary16)][up scales row r], zero padding;
+ *                [gate scales row r (nb_gu binary16), zero padding to a multiple of 16 bytes]
+ *                [up scales row r], zero padding;
  *              down record c at d_off + c*rs_d: [down codes row c][down scales row c];
  *              codes in GGUF block order, Q8_0 codes stored as q + 128 (unsigned byte)
  *   g        device float [top_k] weights of the experts; x device float [hidden], 16-byte

@@ -246,7 +246,7 @@ Layout make_layout(const mf_model_t& m) {
   l.nb_d = (int)(I / 32);
   l.o_up = (uint32_t)l.qrow_gu;
   l.o_gs = 2u * l.qrow_gu;
-  l.o_us = l.o_gs + 2u * l.nb_gu;
+  l.o_us = l.o_gs + ((2u * l.nb_gu + 15) & ~15u);  // 16-byte aligned: the GEMMs load scales by TMA box
   l.rs_gu = (uint32_t)((l.o_us + 2u * l.nb_gu + 15) & ~15u);
   l.o_ds = (uint32_t)l.qrow_d;
   l.rs_d = (uint32_t)((l.qrow_d + 2u * l.nb_d + 15) & ~15u);

@@ -16,8 +16,8 @@ constexpr int kTimerClasses = 7;
 enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5, kTFfn = 6 };
 
 // Layout of one expert slot, identical in the pinned pack and in the HBM pool: row records.
-// Gate/up region: I records, record r = [gate codes row r | up codes row r | gate scales row r
-// | up scales row r], padded to 16 bytes.  Down region: H records, record c = [down codes row c
+// Gate/up region: I records, record r = [gate codes row r | up codes row r | gate scales row r,
+// padded to 16 bytes | up scales row r], padded to 16 bytes.  Down region: H records, record c = [down codes row c
 // | down scales row c], padded to 16 bytes.  Codes: Q8_0 one byte per weight stored as
 // q + 128; Q4_0 the 16 code bytes of each block in GGUF order.  Scales: binary16, one per 32
 // weights.  Rows that are computed together are contiguous, so a work item is one copy.
@@ -188,7 +188,8 @@ struct mf_ctx {
   int prefill_min_t;  // calls with T >= this use the tensor-core grouped GEMMs (0 = never)
   uint8_t* gemm_scratch;  // x and h tiles of the tensor-core path (allocated when first enabled)
   bool tmaps_ok;
-  CUtensorMap tm_gu, tm_d;  // the slot pool's gate/up and down row records as 3-D byte tensors
+  CUtensorMap tm_gu[2], tm_d[2];  // the slot pool's gate/up and down row records as 3-D byte tensors:
+                                  // [0] boxes of one step's codes, [1] boxes of one scale group
 };
 
 namespace mf {
@@ -232,7 +233,7 @@ uint64_t prefill_tiles_max(int T, int k, int E);  // bound on the 128-assignment
 uint64_t prefill_scratch_bytes(int T_max, int k, int E, int hidden, int inter);
 int prefill_tensor_maps(mf_ctx* c);  // encode tm_gu / tm_d for the context's pool; 0 on success
 cudaError_t launch_tile_x(const Dev& d, const float* x, int T, cudaStream_t s);
-cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s);
-cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s);
+cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s);
+cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s);
 
 }  // namespace mf

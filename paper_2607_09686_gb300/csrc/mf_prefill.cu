@@ -99,9 +99,6 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
 // generic-proxy shared-memory writes become visible to the tensor cores' (async proxy) reads
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
-__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
 // 3-D tiled TMA load of a box at (x, y, z) of `tmap` into shared memory, completing on `bar`
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* tmap, int x, int y, int z, uint64_t* bar) {
   asm volatile(
@@ -174,36 +171,47 @@ struct Unit {
 
 // The wave's units, expert by expert: expert u0 + e has ceil(n / 128) assignment blocks times
 // `nrb` row blocks, row blocks innermost (CTAs working on the same assignment block at once
-// share its B tiles in L2).
+// share its B tiles in L2).  Unit i is row block i % nrb of the wave's assignment block i / nrb,
+// found in the exclusive prefix of assignment blocks per unique expert (tb_off).
 struct UnitMap {
   int u0, nu, nrb, total;
-  const int* pre;  // [nu + 1] exclusive prefix of the experts' unit counts
+  const int* tb_off;
   __device__ __forceinline__ Unit at(int i) const {
-    int lo = 0, hi = nu - 1;
-    while (lo < hi) {  // last expert with pre[e] <= i
+    const int ti = __ldg(&tb_off[u0]) + i / nrb;
+    int lo = u0, hi = u0 + nu - 1;
+    while (lo < hi) {  // last expert whose first assignment block is at or before ti
       const int mid = (lo + hi + 1) >> 1;
-      if (pre[mid] <= i) lo = mid;
+      if (__ldg(&tb_off[mid]) <= ti) lo = mid;
       else hi = mid - 1;
     }
-    const int rel = i - pre[lo];
-    return {u0 + lo, rel / nrb, rel % nrb};
+    return {lo, ti - __ldg(&tb_off[lo]), i % nrb};
   }
 };
 
-// Shared memory of one CTA: operand stages, raw ring, barriers, unit prefix.
+// Scales travel in groups of kGroup K steps: one 16-byte TMA box per (tensor, row) holds the
+// group's 8 binary16 scales.  A group's buffer is loaded again two groups later, once the
+// producer has seen the raw slot of a step of the group in between freed; every group but a
+// unit's last has 8 steps and the last has 4 or 8 (K is a multiple of 128), so that step lies
+// inside the group in between whenever the raw ring has at most 4 slots.
+constexpr int kGroup = 8;
+constexpr uint32_t kScaleBox = 16;
+static_assert(kRaw <= 4 && kGroup * 2 == (int)kScaleBox, "scale groups");
+
+// Shared memory of one CTA: operand stages, raw ring, scale ring, barriers.
 template <int NT, int CB>  // tensors per step (2: gate and up, 1: down), code bytes per 32-weight block
 struct PLayout {
-  static constexpr int kNA = 2 * NT;                              // A tiles per stage: hi / lo per tensor
-  static constexpr uint32_t kStage = kNA * kTile + kBTile;        // + B hi / lo
-  static constexpr uint32_t kRawCodes = NT * kBM * CB;            // codes of one step (TMA boxes)
-  static constexpr uint32_t kRawSlot = kRawCodes + NT * kBM * 4;  // + one scale word per (tensor, row)
+  static constexpr int kNA = 2 * NT;                          // A tiles per stage: hi / lo per tensor
+  static constexpr uint32_t kStage = kNA * kTile + kBTile;    // + B hi / lo
+  static constexpr uint32_t kRawSlot = NT * kBM * CB;         // codes of one step (TMA boxes)
+  static constexpr uint32_t kScaleBuf = NT * kBM * kScaleBox;  // scales of one group (TMA boxes)
   static constexpr int kBars = 2 * kRaw + 2 * kStages + 2 * 2 + 1;
   static constexpr uint32_t kOffRaw = kStages * kStage;
-  static constexpr uint32_t kOffBar = kOffRaw + kRaw * kRawSlot;
-  static constexpr uint32_t kOffPre = kOffBar + kBars * 8;
-  static constexpr uint32_t kOffMisc = kOffPre + (kMaxExperts + 1) * 4;
+  static constexpr uint32_t kOffScale = kOffRaw + kRaw * kRawSlot;
+  static constexpr uint32_t kOffBar = kOffScale + 2 * kScaleBuf;
+  static constexpr uint32_t kOffMisc = kOffBar + kBars * 8;
   static constexpr uint32_t kBytes = kOffMisc + 16;
-  static_assert(kRawSlot % 128 == 0 && kOffRaw % 128 == 0, "TMA destinations are 128-byte aligned");
+  static_assert(kRawSlot % 128 == 0 && kOffRaw % 128 == 0 && kOffScale % 128 == 0 && kScaleBuf % 128 == 0,
+                "TMA destinations are 128-byte aligned");
 };
 
 // Gate/up (NT = 2) or down (NT = 1) projection of wave `wave` for every assignment of the wave.
@@ -215,7 +223,8 @@ struct PLayout {
 // epilogue --acc_empty--> MMA, with two TMEM accumulators.
 template <int QT, int NT>
 __global__ void __launch_bounds__(kThreadsW, 1)
-    k_prefill(const __grid_constant__ CUtensorMap tmap, Dev d, int layer, int wave) {
+    k_prefill(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap smap, Dev d, int layer,
+              int wave) {
   constexpr int CB = QT == MF_Q8_0 ? 32 : 16;
   using PL = PLayout<NT, CB>;
   constexpr uint32_t kAcc = NT * kBN;  // TMEM columns of one accumulator (gate | up, or down)
@@ -223,14 +232,13 @@ __global__ void __launch_bounds__(kThreadsW, 1)
   constexpr uint32_t kOffBits = QT == MF_Q8_0 ? dq::kOffQ8 : dq::kOffQ4;
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + PL::kOffBar);
-  uint64_t* full = bars;                    // [kRaw]    32 cp.async arrivals + 1 expect-tx arrival
+  uint64_t* full = bars;                    // [kRaw]    1 expect-tx arrival (codes, scales, B tile)
   uint64_t* raw_free = full + kRaw;         // [kRaw]    one arrival per converter warp
   uint64_t* a_ready = raw_free + kRaw;      // [kStages] one arrival per converter warp
   uint64_t* mma_done = a_ready + kStages;   // [kStages] tcgen05.commit
   uint64_t* acc_full = mma_done + kStages;  // [2]       tcgen05.commit
   uint64_t* acc_empty = acc_full + 2;       // [2]       one arrival per epilogue warp
   uint64_t* drain = acc_empty + 2;          // [1]       tcgen05.commit
-  int* s_pre = reinterpret_cast<int*>(smem + PL::kOffPre);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(smem + PL::kOffMisc);
   volatile int* s_flag = reinterpret_cast<volatile int*>(smem + PL::kOffMisc + 4);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -242,7 +250,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
   // ---- prologue: barriers, tensor memory, the wave's unit prefix
   if (tid == 0) {
     for (int i = 0; i < kRaw; ++i) {
-      mbar_init(&full[i], 33);
+      mbar_init(&full[i], 1);
       mbar_init(&raw_free[i], kConvWarps);
     }
     for (int i = 0; i < kStages; ++i) {
@@ -266,20 +274,12 @@ __global__ void __launch_bounds__(kThreadsW, 1)
   um.u0 = wave * d.S_active;
   um.nu = max(0, min(d.S_active, d.info[0] - um.u0));
   um.nrb = nrb;
-  um.pre = s_pre;
-  if (tid == 32) {
-    int acc = 0;
-    for (int e = 0; e < um.nu; ++e) {
-      s_pre[e] = acc;
-      acc += (d.tb_off[um.u0 + e + 1] - d.tb_off[um.u0 + e]) * nrb;
-    }
-    s_pre[um.nu] = acc;
-  }
+  um.tb_off = d.tb_off;
+  um.total = um.nu > 0 ? (d.tb_off[um.u0 + um.nu] - d.tb_off[um.u0]) * nrb : 0;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem0 = *s_tmem;
-  um.total = s_pre[um.nu];
   const int bid = (int)blockIdx.x, nb = (int)gridDim.x;
   const int n_units = um.total > bid ? (um.total - 1 - bid) / nb + 1 : 0;
   const int n_steps = n_units * nk;
@@ -302,15 +302,21 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     const int ten = NT == 2 ? part : 0, tr = ten * kBM + r;
     constexpr int kGroups = NT == 2 ? 4 : 2;  // 8-weight groups of this thread
     const int g0 = NT == 2 ? 0 : part * 2;
-    int kk = 0, slot = 0, stage = 0;
+    int kk = 0, slot = 0, stage = 0, gb = 1;
     uint32_t rph = 0, sph = 0;  // phase parities of the raw ring and of the stage ring
+    uint4 sv = make_uint4(0, 0, 0, 0);  // this row's scales of the current group
     for (int s = 0; s < n_steps; ++s) {
       if (!warp_wait(&full[slot], rph, 1u)) break;
       if (s >= kStages && !warp_wait(&mma_done[stage], sph ^ 1, 2u)) break;
       const unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
       unsigned char* a_hi = smem + stage * PL::kStage + (2 * ten) * kTile;
       unsigned char* a_lo = a_hi + kTile;
-      const uint32_t sw = *reinterpret_cast<const uint32_t*>(raw + PL::kRawCodes + tr * 4);
+      if ((kk & (kGroup - 1)) == 0) {  // first step of a group: its scales arrived with this step's codes
+        gb ^= 1;
+        sv = *reinterpret_cast<const uint4*>(smem + PL::kOffScale + gb * PL::kScaleBuf + tr * kScaleBox);
+      }
+      const int q = (kk >> 1) & 3;
+      const uint32_t sw = q == 0 ? sv.x : q == 1 ? sv.y : q == 2 ? sv.z : sv.w;
       const float dsc = __half2float(__ushort_as_half((unsigned short)((kk & 1) ? (sw >> 16) : (sw & 0xFFFFu))));
       const uint64_t dd = f2_pack(__float_as_uint(dsc), __float_as_uint(dsc));
       const unsigned char* codes = raw + (size_t)tr * CB;
@@ -351,7 +357,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
     int y0 = 0, z0 = 0;             // its TMA coordinates: first row, slot plane
     size_t b0 = 0;                  // its first B tile
     uint32_t b_bytes = 0;           // bytes of each B half the MMAs read: n_eff columns
-    int kk = 0, slot = 0, stage = 0, j = 0;
+    int kk = 0, slot = 0, stage = 0, j = 0, gb = 1;
     uint32_t rph = 0, sph = 0;
     for (int s = 0; s < n_steps; ++s) {
       if (kk == 0) {
@@ -366,28 +372,32 @@ __global__ void __launch_bounds__(kThreadsW, 1)
       if (s >= kRaw && !warp_wait(&raw_free[slot], rph ^ 1, 3u)) break;
       if (s >= kStages && !warp_wait(&mma_done[stage], sph ^ 1, 4u)) break;
       unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
+      const bool group = (kk & (kGroup - 1)) == 0;
+      if (group) gb ^= 1;
       if (lane == 0) {
-        mbar_arrive_tx(&full[slot], NT * kBM * CB + 2 * b_bytes);
+        mbar_arrive_tx(&full[slot], NT * kBM * CB + 2 * b_bytes + (group ? PL::kScaleBuf : 0u));
 #pragma unroll
         for (int tn = 0; tn < NT; ++tn)
           tma_load_3d(raw + tn * kBM * CB, &tmap, (tn ? (int)d.lay.o_up : 0) + kk * CB, y0, z0, &full[slot]);
+        if (group) {
+          // x = the scale region's start (16-byte aligned in the slot layout) + 16 bytes per group
+#pragma unroll
+          for (int tn = 0; tn < NT; ++tn) {
+            const uint32_t so = NT == 2 ? (tn ? d.lay.o_us : d.lay.o_gs) : d.lay.o_ds;
+            tma_load_3d(smem + PL::kOffScale + gb * PL::kScaleBuf + tn * kBM * kScaleBox, &smap,
+                        (int)(so + (uint32_t)(kk / kGroup) * kScaleBox), y0, z0, &full[slot]);
+          }
+        }
         unsigned char* bdst = smem + stage * PL::kStage + PL::kNA * kTile;
         const uint8_t* bsrc = tiles + (b0 + kk) * kBTile;
         bulk_g2s(bdst, bsrc, b_bytes, &full[slot]);                  // hi: the first n_eff columns
         bulk_g2s(bdst + kTile, bsrc + kTile, b_bytes, &full[slot]);  // lo
       }
-#pragma unroll
-      for (int i = 0; i < NT * kBM / 32; ++i) {
-        const int t = lane + 32 * i, tn = t / kBM, r = t % kBM;
-        const uint32_t so = NT == 2 ? (tn ? d.lay.o_us : d.lay.o_gs) : d.lay.o_ds;
-        cp_async4(raw + PL::kRawCodes + t * 4, rows + (size_t)r * rstride + so + (size_t)(kk & ~1) * 2);
-      }
-      asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_u32(&full[slot])) : "memory");
+      __syncwarp();
       if (++kk == nk) kk = 0, ++j;
       if (++slot == kRaw) slot = 0, rph ^= 1;
       if (++stage == kStages) stage = 0, sph ^= 1;
     }
-    asm volatile("cp.async.wait_all;" ::: "memory");
   } else if (warp == kMmaWarp) {
     // ================= MMA issue (one thread)
     if (lane == 0) {
@@ -539,12 +549,12 @@ int sm_count_p() {
 }
 
 template <int QT, int NT>
-cudaError_t launch_k(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s) {
+cudaError_t launch_k(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s) {
   constexpr size_t smem = PLayout<NT, QT == MF_Q8_0 ? 32 : 16>::kBytes;
   static_assert(smem <= 232448, "shared memory per block");
   cudaError_t e = cudaFuncSetAttribute(k_prefill<QT, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_prefill<QT, NT><<<sm_count_p(), kThreadsW, smem, s>>>(tm, d, layer, wave);
+  k_prefill<QT, NT><<<sm_count_p(), kThreadsW, smem, s>>>(tm[0], tm[1], d, layer, wave);
   return cudaGetLastError();
 }
 
@@ -592,9 +602,12 @@ int prefill_tensor_maps(mf_ctx* c) {
   const Dev& d = c->d;
   const uint32_t cb = d.qtype == MF_Q8_0 ? 32 : 16;
   const uint64_t planes = (uint64_t)d.L * d.S_alloc;
-  if (encode_region(enc, &c->tm_gu, d.pool, d.lay.rs_gu, (uint64_t)d.I, planes, d.lay.stride, cb)) return -1;
-  if (encode_region(enc, &c->tm_d, d.pool + d.lay.d_off, d.lay.rs_d, (uint64_t)d.H, planes, d.lay.stride, cb))
-    return -1;
+  for (int m = 0; m < 2; ++m) {  // code boxes (one step), scale boxes (one group)
+    const uint32_t box = m ? kScaleBox : cb;
+    if (encode_region(enc, &c->tm_gu[m], d.pool, d.lay.rs_gu, (uint64_t)d.I, planes, d.lay.stride, box)) return -1;
+    if (encode_region(enc, &c->tm_d[m], d.pool + d.lay.d_off, d.lay.rs_d, (uint64_t)d.H, planes, d.lay.stride, box))
+      return -1;
+  }
   return 0;
 }
 
@@ -604,11 +617,11 @@ cudaError_t launch_tile_x(const Dev& d, const float* x, int T, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s) {
+cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s) {
   return d.qtype == MF_Q8_0 ? launch_k<MF_Q8_0, 2>(d, tm, layer, wave, s) : launch_k<MF_Q4_0, 2>(d, tm, layer, wave, s);
 }
 
-cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap& tm, int layer, int wave, cudaStream_t s) {
+cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s) {
   return d.qtype == MF_Q8_0 ? launch_k<MF_Q8_0, 1>(d, tm, layer, wave, s) : launch_k<MF_Q4_0, 1>(d, tm, layer, wave, s);
 }
 

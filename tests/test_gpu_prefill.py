@@ -52,9 +52,12 @@ def _boundary_routes(T, E, k, rng):
 
 
 @pytest.mark.parametrize("qtype", [synth.Q8_0, synth.Q4_0])
-def test_gemm_tile_edges_tiny(qtype):
-    """hidden 256, 8 experts, top-4, intermediate 512, 4 slots: 2 waves; counts 256/129/128/127/1."""
-    shape = Shape(1, 256, 8, 4, 512, qtype, model_seed=3)
+@pytest.mark.parametrize("H,I", [(256, 512), (384, 640)])
+def test_gemm_tile_edges_tiny(qtype, H, I):
+    """8 experts, top-4, 4 slots: 2 waves; counts 256/129/128/127/1.  hidden 384 and intermediate
+    640 (K steps 12 and 20) end both GEMMs' reductions on a half scale group, and their 12 gate
+    scales per row are padded to 16 bytes before the up scales."""
+    shape = Shape(1, H, 8, 4, I, qtype, model_seed=3)
     T = 256
     ctx = Ctx(shape, slots=4, max_tokens=T)
     try:

@@ -23,7 +23,7 @@ def slot_image(canon: np.ndarray, H: int, I: int, q: int) -> np.ndarray:
     qgu, qd = (H, I) if q == synth.Q8_0 else (H // 2, I // 2)
     nbgu, nbd = H // 32, I // 32
     o_up, o_gs = qgu, 2 * qgu
-    o_us = o_gs + 2 * nbgu
+    o_us = o_gs + _r(2 * nbgu, 16)
     rs_gu, rs_d = _r(o_us + 2 * nbgu, 16), _r(qd + 2 * nbd, 16)
     d_off = _r(I * rs_gu, 256)
     out = np.zeros(_r(d_off + H * rs_d, 256), np.uint8)
