@@ -34,8 +34,10 @@ N_TOKENS = 256
 
 # DRAM bytes (read + write) of one launch of the roofline kernel (the fused one-token FFN) from
 # the ncu capture summarised under profiles/, valid while the kernel sources hash to `sha`
-# (otherwise the line reports null: the counters no longer describe the kernel that ran).
-KERNEL_TRAFFIC = {"sha": "93e6ef4d9e3953fc", "bytes": 40199424,
+# (otherwise the line reports null: the counters no longer describe the kernel that ran).  The
+# hash is re-recorded without a new capture only when the kernel's compiled device code is
+# byte-identical to the captured build's.
+KERNEL_TRAFFIC = {"sha": "07c0cef5dbf0b6c0", "bytes": 40199424,
                   "files": ("paper_2607_09686_gb300/csrc/mf_decode.cu", "paper_2607_09686_gb300/csrc/mf_dequant.cuh",
                             "paper_2607_09686_gb300/csrc/mf_internal.cuh")}
 

@@ -17,8 +17,8 @@ enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, 
 
 // Layout of one expert slot, identical in the pinned pack and in the HBM pool: row records.
 // Gate/up region: I records, record r = [gate codes row r | up codes row r | gate scales row r,
-// padded to 16 bytes | up scales row r], padded to 16 bytes.  Down region: H records, record c = [down codes row c
-// | down scales row c], padded to 16 bytes.  Codes: Q8_0 one byte per weight stored as
+// padded to 16 bytes | up scales row r], padded to 16 bytes.  Down region: H records, record
+// c = [down codes row c | down scales row c], padded to 16 bytes.  Codes: Q8_0 one byte per weight stored as
 // q + 128; Q4_0 the 16 code bytes of each block in GGUF order.  Scales: binary16, one per 32
 // weights.  Rows that are computed together are contiguous, so a work item is one copy.
 struct Layout {

@@ -22,8 +22,9 @@
 // block), with warp-specialised roles linked by mbarriers:
 //   producer (1 warp)    per step: one TMA load per weight tensor (the 128 rows' codes of the
 //                        block, from a 3-D tensor map over the slot pool) into a 3-slot raw ring,
-//                        cp.async of the 128 rows' scale words, and one bulk copy of the B tile
-//                        into operand stage s % 4;
+//                        every 8 steps one TMA load per tensor of the rows' next 8 scales into a
+//                        2-group scale ring, and one bulk copy of the B tile into operand stage
+//                        s % 4 (lane 0 issues the copies);
 //   converters (8 warps) dequantise the raw codes exactly into the stage's A tiles (hi / lo,
 //                        no-swizzle K-major core-matrix layout): byte -> float by the
 //                        magic-number conversion, times the binary16 scale, split with packed
@@ -350,13 +351,11 @@ __global__ void __launch_bounds__(kThreadsW, 1)
       if (++stage == kStages) stage = 0, sph ^= 1;
     }
   } else if (warp == kProdWarp) {
-    // ================= producer: TMA boxes of codes, cp.async of scale words, bulk B tile
-    const size_t rstride = NT == 2 ? d.lay.rs_gu : d.lay.rs_d;
+    // ================= producer: TMA boxes of codes and scales, bulk B tile
     const uint8_t* tiles = NT == 2 ? d.xt : d.ht;
-    const uint8_t* rows = nullptr;  // the unit's first weight row record
-    int y0 = 0, z0 = 0;             // its TMA coordinates: first row, slot plane
-    size_t b0 = 0;                  // its first B tile
-    uint32_t b_bytes = 0;           // bytes of each B half the MMAs read: n_eff columns
+    int y0 = 0, z0 = 0;    // the unit's TMA coordinates: first row, slot plane
+    size_t b0 = 0;         // its first B tile
+    uint32_t b_bytes = 0;  // bytes of each B half the MMAs read: n_eff columns
     int kk = 0, slot = 0, stage = 0, j = 0, gb = 1;
     uint32_t rph = 0, sph = 0;
     for (int s = 0; s < n_steps; ++s) {
@@ -364,7 +363,6 @@ __global__ void __launch_bounds__(kThreadsW, 1)
         const Unit un = um.at(bid + j * nb);
         z0 = layer * d.S_alloc + d.uslot[un.u];
         y0 = un.rb * kBM;
-        rows = d.pool + (size_t)z0 * d.lay.stride + (NT == 2 ? 0 : d.lay.d_off) + (size_t)y0 * rstride;
         b0 = (size_t)(d.tb_off[un.u] + un.tb) * nk;
         const int a0 = d.asg_off[un.u] + un.tb * kBN;
         b_bytes = (uint32_t)n_eff(min(kBN, d.asg_off[un.u + 1] - a0)) * (kBK * 2);
