@@ -31,6 +31,13 @@ sys.path.insert(0, ROOT)
 
 WORKLOAD = "l4e64"
 N_TOKENS = 256
+METRIC = "MoE-layer decode tokens/s at batch 1 (token = all 4 MoE layers)"  # both arms report it
+
+
+def workload_name(cache_pct: float) -> str:
+    """The headline workload, named the same way by both arms."""
+    return (f"{WORKLOAD}: 4 MoE layers, hidden 2048, 64 experts, top-8, inter 768, Q8_0, "
+            f"256 decode tokens batch 1, Zipf 1.1 + 0.6 reuse, cache {cache_pct:g}%")
 
 # DRAM bytes (read + write) of one launch of the roofline kernel (the fused one-token FFN) from
 # the ncu capture summarised under profiles/, valid while the kernel sources hash to `sha`
@@ -290,7 +297,7 @@ def run_mawforge(args):
     kernels = {name: {"ms_total": round(v[0], 4), "launches": v[1],
                       "us_per_launch": round(1e3 * v[0] / v[1], 3) if v[1] else None} for name, v in kt.items()}
     line = {
-        "metric": "MoE-layer decode tokens/s at batch 1 (token = all 4 MoE layers)",
+        "metric": METRIC,
         "value": round(value, 2),
         "unit": "tokens/s",
         "n_gpus": ws,
@@ -303,8 +310,7 @@ def run_mawforge(args):
         "vs_baseline": None,
         "dtype": "q8_0 weights, f32 activations and accumulation",
         "data": "synthetic (seeded; random-init Q8_0 experts; planted Zipf routing)",
-        "config": {"workload": f"{WORKLOAD}: 4 MoE layers, hidden 2048, 64 experts, top-8, inter 768, Q8_0, "
-                               f"256 decode tokens batch 1, Zipf 1.1 + 0.6 reuse, cache {args.cache_pct:g}%",
+        "config": {"workload": workload_name(args.cache_pct),
                    "cache_pct": args.cache_pct, "slots_per_layer": plan.slots_per_layer,
                    "tokens_per_step": N_TOKENS, "layers": L, "l2": "flushed between steps (512 MB write)",
                    "execution": "one CUDA graph per step of the 1024 C-ABI calls"},
@@ -352,7 +358,7 @@ def run_mawforge(args):
     if not args.no_batch64 and rank == 0:
         line["batch64"] = batch64_measurement(torch, mf, synth, device)
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        runs = [cpu_baseline(args.cpu_tokens) for _ in range(args.cpu_passes)]
+        runs = [cpu_baseline(args.cpu_tokens, args.cache_pct) for _ in range(args.cpu_passes)]
         line["cpu_baseline"] = dict(runs[0], value=round(statistics.mean(r["value"] for r in runs), 4),
                                     sample=runs[0]["sample"] + f", {args.cpu_passes} passes from a cold cache")
     if rank == 0:
@@ -576,15 +582,16 @@ def _bf16_peak():
         return 1900.0, "fallback"
 
 
-def cpu_baseline(n_tokens: int) -> dict:
-    """The CPU oracle, as it stands, on the first tokens of the same workload."""
+def cpu_baseline(n_tokens: int, cache_pct: float = 35.0) -> dict:
+    """The CPU oracle, as it stands, on the first tokens of the same workload (same cache share)."""
     import oracle
     import synth
     cfg = synth.CONFIGS[WORKLOAD]
     L, H, E, k, I, q = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
     route = cfg.route_classes[0]
     pays = {}
-    lru = [oracle.LRU(E, int(np.floor(35.0 * E / 100 + 1e-9)), synth.payload_bytes(H, I, q)) for _ in range(L)]
+    slots = max(k, int(np.floor(cache_pct * E / 100 + 1e-9)))  # the planner's slot count
+    lru = [oracle.LRU(E, slots, synth.payload_bytes(H, I, q)) for _ in range(L)]
     xs = [synth.activations(0, l, 0, 0, n_tokens, H) for l in range(L)]
     bs = [synth.plant_bias(synth.routes(0, l, 0, E, k, n_tokens, route.zipf_s, route.reuse), E) for l in range(L)]
     wrs = [synth.router_weights(cfg.model_seed, l, E, H) for l in range(L)]
@@ -600,8 +607,9 @@ def cpu_baseline(n_tokens: int) -> dict:
     dt = time.perf_counter() - t0
     cores = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     return {"value": round(n_tokens / dt, 4), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "slots_per_layer": slots,
             "sample": f"first {n_tokens} tokens of the same sequence (256 = the whole step), all {L} layers "
-                      "(router + LRU + fp64 layer)"}
+                      f"(router + LRU with {slots} slots + fp64 layer)"}
 
 
 def run_reference(args):
@@ -610,15 +618,16 @@ def run_reference(args):
         return
     per_step = []
     for i in range(args.warmup + args.steps):
-        r = cpu_baseline(args.cpu_tokens)
+        r = cpu_baseline(args.cpu_tokens, getattr(args, "cache_pct", 35.0))
         if i >= args.warmup:
             per_step.append(r)
     value = statistics.mean(r["value"] for r in per_step)
-    line = {"impl": "reference", "metric": "MoE-layer decode tokens/s at batch 1 (token = all 4 MoE layers)",
+    line = {"impl": "reference", "metric": METRIC,
             "value": round(value, 4), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(1e3 * args.cpu_tokens / value, 3), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64 (CPU oracle)", "data": "synthetic (seeded)",
-            "config": {"workload": f"{WORKLOAD} (the same workload; a bounded sample of it per step)",
+            "config": {"workload": workload_name(getattr(args, "cache_pct", 35.0)),
+                       "sample": f"the first {args.cpu_tokens} tokens of the 256-token step",
                        "tokens_per_step": args.cpu_tokens},
             "cpu_baseline": {"value": round(value, 4), "unit": "tokens/s", "kind": "oracle",
                              "cores": per_step[0]["cores"], "sample": per_step[0]["sample"]},
