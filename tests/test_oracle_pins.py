@@ -125,6 +125,29 @@ def test_router_ties_go_to_lower_expert_and_equal_weights():
     assert list(idx) == [7, 1, 2, 4]
 
 
+def test_router_weights_are_full_softmax_renormalised_over_the_selection():
+    """Softmax over the k selected logits equals a library softmax over all E logits followed by
+    renormalisation over the same k (the weights of the routed experts, section "Native Serving
+    Path"); a gap of thousands between the first two logits gives weights (1, 0, ...) without
+    overflow."""
+    from scipy.special import softmax
+    rng = np.random.default_rng(12)
+    E, H, k = 16, 48, 4
+    wr = (rng.standard_normal((E, H)) * 0.02).astype(np.float32)
+    for trial in range(10):
+        x = rng.standard_normal(H).astype(np.float32)
+        bias = (rng.standard_normal(E) * 2.0).astype(np.float32)
+        z, idx, g = oracle.router(x, wr, bias, k)
+        full = softmax(z.astype(np.float64))
+        ref = full[idx] / full[idx].sum()
+        assert np.allclose(g, ref, rtol=1e-12, atol=0)
+    bias = np.zeros(E, np.float32)
+    bias[3], bias[9] = 4000.0, 1000.0
+    z, idx, g = oracle.router(np.zeros(H, np.float32), wr, bias, 2)
+    assert list(idx) == [3, 9]
+    assert g[0] == 1.0 and g[1] == 0.0 and np.isfinite(g).all()
+
+
 # ---------------------------------------------------------------- expert FFN and layer
 def _silu(v):
     return v / (1.0 + np.exp(-v))
