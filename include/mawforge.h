@@ -98,6 +98,40 @@ typedef struct mf_ctx mf_ctx_t;
 /* Canonical GGUF bytes of one expert payload.  Host only. */
 int mf_payload_bytes(const mf_model_t* model, uint64_t* out);
 
+/* One candidate cache size of mf_tune_cache. */
+typedef struct mf_tune_point {
+  double cache_pct;                 /* the candidate p (copied from the request) */
+  int32_t accepted, slots_per_layer; /* mf_plan's decision and S for p */
+  uint64_t pool_bytes, footprint_bytes;
+  uint64_t accesses, hits, misses;  /* the trace replayed through per-layer caches of S slots */
+  uint64_t bytes_materialized;      /* misses * payload_bytes */
+  double predicted_s;               /* n_tokens * t_token_s + misses * t_miss_s */
+  double predicted_tokens_per_s;    /* n_tokens / predicted_s (0 when predicted_s is 0) */
+} mf_tune_point_t;
+
+/* Cache-size tuner (section "Throughput Model": T(p) = tokens / (compute_time +
+ * materialization_time(p) + pressure_penalty(F)); Discussion, "Cache Hit Rate Is an Incomplete
+ * Objective": choose the cache point that minimises end-to-end latency under the memory budget,
+ * not the one that maximises hit rate).  Host only, no GPU needed.
+ *   routes    host int32 [n_layers][n_tokens][top_k]: a route trace (expert ids in [0,
+ *             n_experts), each token's in the router's rank order, as idx_out returns them: the
+ *             order the cache sees), replayed layer by layer in steps of T consecutive tokens
+ *             (the last step may be shorter), with the library's cache semantics: per step the
+ *             distinct experts in the given access order (MF_ORDER_*), least-recently-used
+ *             replacement
+ *   t_token_s measured seconds per token with every expert resident (all layers);
+ *   t_miss_s  measured seconds per materialised payload (the link's share of a miss)
+ *   pcts      host [n] candidate cache percentages; req supplies the other plan inputs
+ *   out       host [n] results, in the order of pcts; *best = the accepted candidate with the
+ *             highest predicted rate (ties: the smaller pool, then the earlier candidate), or -1
+ * The pressure term is zero: on a GB300 the slot pool is dedicated HBM, so a plan inside the
+ * static budget pages nothing.  MF_E_INVAL for NULL pointers, n < 1, n_tokens < 1, T < 1, an
+ * expert id out of range, negative or non-finite times, an unknown order or an invalid p;
+ * MF_E_BUDGET (with out and *best = -1 filled) when no candidate is accepted. */
+int mf_tune_cache(const mf_model_t* model, const mf_plan_req_t* req, const int32_t* routes, int n_tokens, int T,
+                  int order, double t_token_s, double t_miss_s, const double* pcts, int n, mf_tune_point_t* out,
+                  int* best);
+
 /* Static budget check (section "Static Budget Check").  Host-only arithmetic, no GPU
  * needed.  Fills *out even when rejecting; returns MF_E_BUDGET if L > budget. */
 int mf_plan(const mf_model_t* model, const mf_plan_req_t* req, mf_plan_t* out);
@@ -158,8 +192,8 @@ int mf_prefill_threshold(mf_ctx_t* ctx, int min_tokens);
  * first-occurrence order.  MF_ORDER_RESIDENT_FIRST: the experts that are resident when the
  * call starts come first (in first-occurrence order among themselves), then the others (in
  * first-occurrence order): every one of them hits, whereas in first-occurrence order an early
- * miss can evict an expert the same step needs later.  Calls with T = 1 are unaffected (their k
- * distinct experts form one wave, and no access of a wave evicts another of it).  Waves,
+ * miss can evict an expert the same step needs later.  Calls with T = 1 keep first-occurrence
+ * order whatever is set (the order applies to calls with T > 1 only).  Waves,
  * counters, traces and outputs follow the chosen order.  MF_E_INVAL for any other value.  Host
  * only; applies to calls issued afterwards. */
 int mf_access_order(mf_ctx_t* ctx, int order);

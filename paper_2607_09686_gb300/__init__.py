@@ -15,8 +15,8 @@ import ctypes
 import os
 
 __all__ = [
-    "MFError", "Model", "PlanReq", "Plan", "Stats", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
-    "mf_payload_bytes", "mf_plan", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
+    "MFError", "Model", "PlanReq", "Plan", "Stats", "TunePoint", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
+    "mf_payload_bytes", "mf_plan", "mf_tune_cache", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
     "mf_moe_forward_host", "mf_prefill_threshold", "mf_access_order", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_expert_ffn_noalloc", "mf_destroy",
     "mf_strerror", "mf_last_cuda_error",
 ]
@@ -61,10 +61,22 @@ class Stats(ctypes.Structure):
         return {name: int(getattr(self, name)) for name, _ in self._fields_}
 
 
+class TunePoint(ctypes.Structure):
+    _fields_ = [("cache_pct", ctypes.c_double), ("accepted", ctypes.c_int32), ("slots_per_layer", ctypes.c_int32),
+                ("pool_bytes", ctypes.c_uint64), ("footprint_bytes", ctypes.c_uint64), ("accesses", ctypes.c_uint64),
+                ("hits", ctypes.c_uint64), ("misses", ctypes.c_uint64), ("bytes_materialized", ctypes.c_uint64),
+                ("predicted_s", ctypes.c_double), ("predicted_tokens_per_s", ctypes.c_double)]
+
+    def as_dict(self) -> dict:
+        return {name: getattr(self, name) for name, _ in self._fields_}
+
+
 _vp, _i32, _u64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_uint64
 _sig = {
     "mf_payload_bytes": (_i32, [ctypes.POINTER(Model), ctypes.POINTER(_u64)]),
     "mf_plan": (_i32, [ctypes.POINTER(Model), ctypes.POINTER(PlanReq), ctypes.POINTER(Plan)]),
+    "mf_tune_cache": (_i32, [ctypes.POINTER(Model), ctypes.POINTER(PlanReq), _vp, _i32, _i32, _i32, ctypes.c_double,
+                             ctypes.c_double, _vp, _i32, ctypes.POINTER(TunePoint), ctypes.POINTER(_i32)]),
     "mf_create": (_i32, [ctypes.POINTER(_vp), ctypes.POINTER(Model), ctypes.POINTER(Plan), _i32]),
     "mf_pack_put": (_i32, [_vp, _i32, _i32, _vp, _u64]),
     "mf_load_pack": (_i32, [ctypes.POINTER(_vp), ctypes.POINTER(Model), ctypes.POINTER(Plan), _vp, _i32]),
@@ -145,6 +157,25 @@ def mf_plan(model: Model, req: PlanReq) -> Plan:
     if rc not in (MF_OK, MF_E_BUDGET):
         _check(rc, "mf_plan")
     return out
+
+
+def mf_tune_cache(model: Model, req: PlanReq, routes, T: int, t_token_s: float, t_miss_s: float, pcts,
+                  order: int = 0):
+    """Cache-size tuner (host only).  routes: int32 array [n_layers][n_tokens][top_k] (C order).
+    Returns (list of per-candidate dicts, index of the best accepted candidate or -1)."""
+    import numpy as np
+    r = np.ascontiguousarray(routes, dtype=np.int32)
+    if r.ndim != 3:
+        raise ValueError("routes must be [n_layers][n_tokens][top_k]")
+    n = len(pcts)
+    cand = (ctypes.c_double * max(1, n))(*[float(p) for p in pcts])
+    out = (TunePoint * max(1, n))()
+    best = _i32(-1)
+    rc = _lib.mf_tune_cache(ctypes.byref(model), ctypes.byref(req), r.ctypes.data, r.shape[1], T, order,
+                            float(t_token_s), float(t_miss_s), cand, n, out, ctypes.byref(best))
+    if rc not in (MF_OK, MF_E_BUDGET):
+        _check(rc, "mf_tune_cache")
+    return [out[i].as_dict() for i in range(n)], best.value
 
 
 def mf_create(model: Model, plan: Plan, device: int = 0) -> int:
