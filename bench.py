@@ -357,6 +357,11 @@ def run_mawforge(args):
         line["prefill"] = prefill_measurement(torch, mf, synth, device)
     if not args.no_batch64 and rank == 0:
         line["batch64"] = batch64_measurement(torch, mf, synth, device)
+    if not args.no_tuner and rank == 0:  # last of the GPU measurements: a failure here costs only this object
+        try:
+            line["tuner"] = tuner_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, h2d)
+        except Exception as e:
+            line["tuner"] = {"error": f"{type(e).__name__}: {e}"}
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         runs = [cpu_baseline(args.cpu_tokens, args.cache_pct) for _ in range(args.cpu_passes)]
         line["cpu_baseline"] = dict(runs[0], value=round(statistics.mean(r["value"] for r in runs), 4),
@@ -417,6 +422,94 @@ def resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, s
             "misses_in_timed_replays": st["misses"],
             "how": "same calls, 100 % cache warmed by two passes (every launch all-resident), L2 flushed per replay",
             "read_floor": read_floor(torch, device, stream, flush, bytes_per_launch, hbm)}
+
+
+def tuner_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, h2d_gbs: float,
+                      pcts=(15.0, 25.0, 35.0, 50.0, 100.0), reps: int = 3) -> dict:
+    """The cache-size tuner (mf_tune_cache) against measured steps of the same workload.  One
+    context with a 100 % pool: a cold pass records the route trace (the router's output order),
+    a warm pass makes every expert resident and its graph replays give the all-resident time per
+    token; with the pinned link rate per payload these go into the tuner.  Each candidate size is
+    then run (mf_reset to its slot count, graph replays that start cold) and its measured rate
+    and miss count set beside the tuner's prediction."""
+    cfg = synth.CONFIGS[WORKLOAD]
+    L, H, E, k, I, q = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    model = mf.Model(L, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(100.0, 1 << 62, 0, 0, 1, 0))
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    try:
+        buf = np.empty(plan.payload_bytes, np.uint8)
+        for l in range(L):
+            for e in range(E):
+                synth.payload(cfg.model_seed, l, e, H, I, q, out=buf)
+                mf.mf_pack_put(ctx, l, e, buf)
+        y = torch.empty(N_TOKENS, L, H, device=device)
+        idx = torch.empty(N_TOKENS, L, k, dtype=torch.int32, device=device)
+
+        def calls(reset: bool, record: bool = False):
+            if reset:
+                mf.mf_reset(ctx, 0, stream)
+            for t in range(N_TOKENS):
+                for l in range(L):
+                    mf.mf_moe_forward(ctx, l, x[t, l], wr[l], bias[t, l], 1, y[t, l], idx[t, l] if record else None,
+                                      None, stream)
+
+        def replay_ms(graph) -> float:  # one untimed replay, then the mean of `reps` (L2 flushed before each)
+            ms = []
+            for i in range(1 + reps):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                with torch.cuda.stream(stream):
+                    flush.zero_()
+                    a.record(stream)
+                    graph.replay()
+                    b.record(stream)
+                torch.cuda.synchronize()
+                if i:
+                    ms.append(a.elapsed_time(b))
+            return statistics.mean(ms)
+
+        with torch.cuda.stream(stream):
+            calls(True, record=True)  # cold: the routes as the cache sees them
+            calls(False)  # warm: every expert of the sequence resident
+            stream.synchronize()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                calls(False)
+        torch.cuda.synchronize()
+        routes = idx.permute(1, 0, 2).contiguous().cpu().numpy()  # [L][tokens][k]
+        resident_ms = replay_ms(g)
+        del g
+        t_token = resident_ms * 1e-3 / N_TOKENS
+        t_miss = plan.payload_bytes / (h2d_gbs * 1e9)
+        pts, best = mf.mf_tune_cache(model, mf.PlanReq(0.0, 1 << 62, 0, 0, 1, 0), routes, 1, t_token, t_miss,
+                                     list(pcts))
+        points = []
+        for pt in pts:
+            mf.mf_reset(ctx, pt["slots_per_layer"], stream)
+            with torch.cuda.stream(stream):
+                calls(True)
+                stream.synchronize()
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=stream):
+                    calls(True)
+            torch.cuda.synchronize()
+            ms = replay_ms(g)
+            del g
+            st = mf.mf_stats(ctx, -1)  # the last replay's counters: every replay starts with a reset
+            points.append({"cache_pct": pt["cache_pct"], "slots_per_layer": pt["slots_per_layer"],
+                           "misses_predicted": pt["misses"], "misses_measured": st["misses"],
+                           "tokens_per_s_predicted": round(pt["predicted_tokens_per_s"], 1),
+                           "tokens_per_s_measured": round(N_TOKENS / (ms * 1e-3), 1)})
+        assert mf.mf_check(ctx) == 0
+    finally:
+        mf.mf_destroy(ctx)
+    measured_best = max(range(len(points)), key=lambda i: points[i]["tokens_per_s_measured"])
+    return {"how": "route trace of the 1024 calls (router order), all-resident time per token from graph replays "
+                   "of a warm 100 % cache, link time per payload at the measured pinned copy rate; each candidate "
+                   "run from a cold cache of its slot count (one context, mf_reset), L2 flushed per replay",
+            "t_token_us": round(t_token * 1e6, 3), "t_miss_us": round(t_miss * 1e6, 3),
+            "points": points, "best_predicted_pct": pts[best]["cache_pct"] if best >= 0 else None,
+            "best_measured_pct": points[measured_best]["cache_pct"]}
 
 
 def h2d_bandwidth(torch, device, stream, nbytes: int = 1 << 30, reps: int = 3) -> float:
@@ -648,6 +741,7 @@ def main():
     ap.add_argument("--no-prefill", action="store_true", help="skip the 4096-token prefill measurement")
     ap.add_argument("--no-resident", action="store_true", help="skip the all-resident FFN measurement")
     ap.add_argument("--no-batch64", action="store_true", help="skip the 64-stream batched decode measurement")
+    ap.add_argument("--no-tuner", action="store_true", help="skip the cache-size tuner against measured steps")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle
