@@ -362,6 +362,12 @@ def run_mawforge(args):
             line["tuner"] = tuner_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, h2d)
         except Exception as e:
             line["tuner"] = {"error": f"{type(e).__name__}: {e}"}
+    if not args.no_spec and rank == 0:
+        try:
+            line["speculative"] = spec_measurement(torch, mf, synth, device, x, bias, wr, stream, flush,
+                                                   args.cache_pct)
+        except Exception as e:
+            line["speculative"] = {"error": f"{type(e).__name__}: {e}"}
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         runs = [cpu_baseline(args.cpu_tokens, args.cache_pct) for _ in range(args.cpu_passes)]
         line["cpu_baseline"] = dict(runs[0], value=round(statistics.mean(r["value"] for r in runs), 4),
@@ -510,6 +516,97 @@ def tuner_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, h2d_
             "t_token_us": round(t_token * 1e6, 3), "t_miss_us": round(t_miss * 1e6, 3),
             "points": points, "best_predicted_pct": pts[best]["cache_pct"] if best >= 0 else None,
             "best_measured_pct": points[measured_best]["cache_pct"]}
+
+
+def spec_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, cache_pct: float, K: int = 4,
+                     alpha: float = 0.6, reps: int = 2) -> dict:
+    """Verification-width accounting of speculative decoding on the same 256 tokens (section
+    "Throughput Model": extra_materialization; Discussion: record drafted and accepted tokens,
+    verification width, misses and materialised bytes).  No draft model: a seeded schedule
+    accepts the first a of K drafts per verify step (each with probability alpha), and rejected
+    drafts carry routes and activations of an independent stream.  Each verify step is one call
+    per layer with T = K + 1 (the union of its rows' experts is materialised); plain decode is
+    one call per token and layer.  Both run eagerly on one context from a cold cache, CUDA
+    events around the whole sequence; the cache-size tuner replays each recorded trace to
+    predict its misses."""
+    cfg = synth.CONFIGS[WORKLOAD]
+    L, H, E, k, I, q = cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    route = cfg.route_classes[0]
+    W = K + 1
+    rows = synth.verify_rows(0, N_TOKENS, K, alpha)  # [batches, W]
+    nb, n_drafts = rows.shape[0], int((rows < 0).sum())
+    xh, bh = x.cpu().numpy(), bias.cpu().numpy()  # [T, L, H], [T, L, E]
+    xb = np.empty((nb, L, W, H), np.float32)
+    bb = np.empty((nb, L, W, E), np.float32)
+    for l in range(L):
+        xd = synth.activations(0, l, 1, 0, n_drafts, H)
+        bd = synth.plant_bias(synth.routes(0, l, 1, E, k, n_drafts, route.zipf_s, 0.0), E)
+        for b in range(nb):
+            for j in range(W):
+                v = int(rows[b, j])
+                xb[b, l, j] = xh[v, l] if v >= 0 else xd[-1 - v]
+                bb[b, l, j] = bh[v, l] if v >= 0 else bd[-1 - v]
+    xb, bb = torch.from_numpy(xb).to(device), torch.from_numpy(bb).to(device)
+    model = mf.Model(L, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(cache_pct, 1 << 62, 0, 0, W, 0))
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    try:
+        buf = np.empty(plan.payload_bytes, np.uint8)
+        for l in range(L):
+            for e in range(E):
+                synth.payload(cfg.model_seed, l, e, H, I, q, out=buf)
+                mf.mf_pack_put(ctx, l, e, buf)
+        y1 = torch.empty(N_TOKENS, L, H, device=device)
+        yb = torch.empty(nb, L, W, H, device=device)
+        i1 = torch.empty(N_TOKENS, L, k, dtype=torch.int32, device=device)
+        ib = torch.empty(nb, L, W, k, dtype=torch.int32, device=device)
+
+        def decode():
+            for t in range(N_TOKENS):
+                for l in range(L):
+                    mf.mf_moe_forward(ctx, l, x[t, l], wr[l], bias[t, l], 1, y1[t, l], i1[t, l], None, stream)
+
+        def verify():
+            for b in range(nb):
+                for l in range(L):
+                    mf.mf_moe_forward(ctx, l, xb[b, l], wr[l], bb[b, l], W, yb[b, l], ib[b, l], None, stream)
+
+        def run(fn):  # one untimed pass, then the mean of `reps`; each from a cold cache
+            ms = []
+            for i in range(1 + reps):
+                with torch.cuda.stream(stream):
+                    flush.zero_()
+                    mf.mf_reset(ctx, 0, stream)
+                    a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record(stream)
+                    fn()
+                    z.record(stream)
+                z.synchronize()
+                if i:
+                    ms.append(a.elapsed_time(z))
+            return statistics.mean(ms), mf.mf_stats(ctx, -1)
+
+        ms1, st1 = run(decode)
+        msv, stv = run(verify)
+        assert mf.mf_check(ctx) == 0
+        tr1 = i1.permute(1, 0, 2).contiguous().cpu().numpy()  # [L][tokens][k]
+        trv = ib.permute(1, 0, 2, 3).reshape(L, nb * W, k).contiguous().cpu().numpy()  # [L][rows][k]
+    finally:
+        mf.mf_destroy(ctx)
+    req = mf.PlanReq(0.0, 1 << 62, 0, 0, W, 0)
+    p1 = mf.mf_tune_cache(model, req, tr1, 1, 0.0, 0.0, [cache_pct])[0][0]
+    pv = mf.mf_tune_cache(model, req, trv, W, 0.0, 0.0, [cache_pct])[0][0]
+    return {"how": "seeded acceptance schedule (no draft model), verify steps of K + 1 rows as one call per "
+                   "layer, plain decode as one call per token and layer, eager calls on one context from a "
+                   "cold cache, CUDA events around each whole sequence",
+            "K": K, "alpha": alpha, "width": W, "cache_pct": cache_pct, "tokens": N_TOKENS, "verify_steps": nb,
+            "accepted_drafts": N_TOKENS - nb, "rejected_drafts": n_drafts,
+            "misses": {"decode": st1["misses"], "decode_predicted": p1["misses"],
+                       "verify": stv["misses"], "verify_predicted": pv["misses"]},
+            "extra_materialized_mb_per_token": round((stv["bytes_materialized"] - st1["bytes_materialized"])
+                                                     / N_TOKENS / 1e6, 3),
+            "tokens_per_s": {"decode": round(N_TOKENS / (ms1 * 1e-3), 1),
+                             "speculative": round(N_TOKENS / (msv * 1e-3), 1)}}
 
 
 def h2d_bandwidth(torch, device, stream, nbytes: int = 1 << 30, reps: int = 3) -> float:
@@ -742,6 +839,7 @@ def main():
     ap.add_argument("--no-resident", action="store_true", help="skip the all-resident FFN measurement")
     ap.add_argument("--no-batch64", action="store_true", help="skip the 64-stream batched decode measurement")
     ap.add_argument("--no-tuner", action="store_true", help="skip the cache-size tuner against measured steps")
+    ap.add_argument("--no-spec", action="store_true", help="skip the speculative verification-width accounting")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle

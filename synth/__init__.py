@@ -63,6 +63,8 @@ def _lib():
         lib.syn_permutation.argtypes = [u64, i32, i32, vp]
         lib.syn_routes.restype = i32
         lib.syn_routes.argtypes = [u64, i32, i32, i32, i32, i32, dbl, dbl, vp]
+        lib.syn_accepts.restype = i32
+        lib.syn_accepts.argtypes = [u64, i32, i32, i32, dbl, vp]
         _LIB = lib
     return _LIB
 
@@ -134,3 +136,34 @@ def plant_bias(route_sets: np.ndarray, n_experts: int) -> np.ndarray:
     rows = np.repeat(np.arange(n), k)
     bias[rows, route_sets.reshape(-1)] = np.tile(16.0 + (k - ranks) * 0.5, n)
     return bias
+
+
+def accepts(seed: int, stream: int, n_steps: int, K: int, alpha: float) -> np.ndarray:
+    """[n_steps] drafted tokens accepted per verify step (leading successes, probability alpha each)."""
+    out = np.empty(n_steps, dtype=np.int32)
+    if _lib().syn_accepts(seed, stream, n_steps, K, float(alpha), out.ctypes.data):
+        raise ValueError("bad schedule parameters")
+    return out
+
+
+def verify_rows(seed: int, n_tokens: int, K: int, alpha: float) -> np.ndarray:
+    """Rows of the verify batches of a speculative run over n_tokens tokens: [n_batches, K + 1].
+    Batch i starts at the first uncommitted token p_i and holds K + 1 rows: the tokens p_i ..
+    p_i + a_i (the target's own token and the a_i accepted drafts) and then rejected drafts;
+    p_{i+1} = p_i + a_i + 1.  Entry >= 0: that token of the sequence; entry < 0: rejected draft
+    number -1 - entry (numbered from 0 across the run).  Rows past the sequence's end are drafts."""
+    acc = accepts(seed, 0, n_tokens, K, alpha)  # every step commits at least one token
+    rows, p, drafts, i = [], 0, 0, 0
+    while p < n_tokens:
+        a = int(acc[i])
+        row = []
+        for j in range(K + 1):
+            if j <= a and p + j < n_tokens:
+                row.append(p + j)
+            else:
+                row.append(-1 - drafts)
+                drafts += 1
+        rows.append(row)
+        p += a + 1
+        i += 1
+    return np.array(rows, dtype=np.int32).reshape(-1, K + 1)

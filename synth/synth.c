@@ -207,3 +207,21 @@ int syn_routes(uint64_t seed, int layer, int stream, int n_experts, int top_k, i
   }
   return 0;
 }
+
+/*
+ * Speculative verification schedule (the workload of a verify-width study; no draft model):
+ * verify step i checks K drafted tokens and the target accepts the first a_i of them, a_i =
+ * the number of leading successes of independent trials that each succeed with probability
+ * alpha (trial j of step i: value j of the stream of domain 6, step i).  The same schedule
+ * serves every layer.  out[i] = a_i in [0, K].
+ */
+int syn_accepts(uint64_t seed, int stream, int n_steps, int K, double alpha, int32_t* out) {
+  if (n_steps < 0 || K < 0 || !(alpha >= 0.0 && alpha <= 1.0)) return -1;
+  for (int i = 0; i < n_steps; ++i) {
+    const uint64_t key = syn_key(seed, 6, (uint64_t)stream, (uint64_t)i, 0);
+    int a = 0;
+    while (a < K && unif(draw(key, (uint64_t)a)) < alpha) ++a;
+    out[i] = a;
+  }
+  return 0;
+}

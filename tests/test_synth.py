@@ -70,3 +70,40 @@ def test_plant_bias_orders_the_set():
     r = np.array([[5, 2, 7]], np.int32)
     b = synth.plant_bias(r, 8)
     assert b[0, 5] == 17.5 and b[0, 2] == 17.0 and b[0, 7] == 16.5 and b[0].sum() == 51.0
+
+
+def test_acceptance_schedule_extremes_and_mean():
+    """a_i counts the leading successes of K trials of probability alpha: 0 for alpha = 0, K for
+    alpha = 1, and mean sum_{j=1..K} alpha^j (a truncated geometric count) over many steps."""
+    assert (synth.accepts(1, 0, 500, 4, 0.0) == 0).all()
+    assert (synth.accepts(1, 0, 500, 4, 1.0) == 4).all()
+    assert (synth.accepts(1, 0, 50, 0, 0.7) == 0).all()
+    n, K, alpha = 40000, 4, 0.6
+    a = synth.accepts(7, 0, n, K, alpha)
+    assert a.min() >= 0 and a.max() <= K
+    mean = sum(alpha ** j for j in range(1, K + 1))
+    var = sum((2 * j - 1) * alpha ** j for j in range(1, K + 1)) - mean ** 2  # E[a^2] = sum (2j-1) P(a >= j)
+    assert abs(a.mean() - mean) < 4 * (var / n) ** 0.5
+    assert np.array_equal(a, synth.accepts(7, 0, n, K, alpha))
+    assert not np.array_equal(a[:100], synth.accepts(8, 0, 100, K, alpha))
+
+
+@pytest.mark.parametrize("K,alpha", [(4, 0.6), (2, 0.0), (3, 1.0), (0, 0.5)])
+def test_verify_rows_cover_the_sequence_once(K, alpha):
+    """Every token appears once, in order, as a prefix of its batch (the target's token and the
+    accepted drafts); the rest of each batch are rejected drafts numbered 0, 1, ... in order;
+    K = 0 is plain decode."""
+    n = 97
+    rows = synth.verify_rows(3, n, K, alpha)
+    assert rows.shape[1] == K + 1
+    toks = [int(v) for v in rows.reshape(-1) if v >= 0]
+    assert toks == list(range(n))
+    drafts = [int(-1 - v) for v in rows.reshape(-1) if v < 0]
+    assert drafts == list(range(len(drafts)))
+    acc = synth.accepts(3, 0, n, K, alpha)
+    for i, row in enumerate(rows):
+        m = int((row >= 0).sum())
+        assert (row[:m] >= 0).all() and (row[m:] < 0).all()
+        assert m == min(int(acc[i]) + 1, n - int(row[0]))
+    if K == 0:
+        assert rows.reshape(-1).tolist() == list(range(n))
