@@ -163,3 +163,31 @@ def test_none_accepted_and_bad_arguments(mf):
     assert call(pcts=())[0] == -1
     assert call(pcts=(101.0,))[0] == -1
     assert call(model=mf.Model(1, 200, E, k, 512, mf.Q8_0))[0] == -1
+
+
+def test_batched_workload_under_its_pool_cap(mf):
+    """The 30-layer, 64-stream workload (128 experts, top-8) under a 12 GiB slot-pool cap with
+    the router weights resident: the static check accepts 15 % only, so the choice is 15 %
+    whatever the rates; 64-token steps (about a hundred distinct experts each against 19 slots)
+    replay like the oracle in both access orders (4 layers of the trace, 8 steps)."""
+    c = synth.CONFIGS["l30e128b64"]
+    L, E, k, B = 4, c.n_experts, c.top_k, c.batch
+    common = c.n_layers * E * c.hidden * 4
+    model = mf.Model(c.n_layers, c.hidden, E, k, c.inter, c.qtype)
+    req = mf.PlanReq(0.0, 12 * 2**30, common, 0, B, 0)
+    routes = np.zeros((c.n_layers, 8 * B, k), np.int32)
+    for l in range(L):  # 64 independent streams per step, Zipf 1.0, stream-major within a step
+        streams = [synth.routes(0, l, s, E, k, 8, 1.0, 0.0) for s in range(B)]
+        for step in range(8):
+            for s in range(B):
+                routes[l, step * B + s] = streams[s][step]
+    routes[L:] = routes[:1]  # layers 4..29 repeat layer 0's trace
+    pcts = [15.0, 35.0, 50.0, 75.0]
+    for order in (0, 1):
+        pts, best = mf.mf_tune_cache(model, req, routes, B, 1e-4, 1e-3, pcts, order)
+        assert [bool(p["accepted"]) for p in pts] == [True, False, False, False]
+        assert best == 0 and pts[0]["slots_per_layer"] == 19
+        for pt in pts:
+            S = pt["slots_per_layer"]
+            exp = _oracle_replay(routes, E, S, B, order)
+            assert (pt["accesses"], pt["hits"], pt["misses"]) == exp, (order, pt["cache_pct"])
