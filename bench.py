@@ -62,6 +62,9 @@ def _captured_traffic():
     return KERNEL_TRAFFIC["bytes"] if KERNEL_TRAFFIC["sha"] == _sources_sha() else None
 
 
+HBM_NOMINAL_GBS = 8000.0  # the GPU's nominal HBM3e bandwidth (~8 TB/s), reported beside the measured copy peak
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -320,6 +323,7 @@ def run_mawforge(args):
         "roofline": {"bound": "hbm", "kernel": rf_kernel,
                      "achieved": round(rf_gbs, 1), "peak": hbm, "unit": "GB/s",
                      "frac": round(rf_gbs / hbm, 4), "peak_kind": peak_kind, "traffic": _captured_traffic(),
+                     "frac_of_nominal": round(rf_gbs / HBM_NOMINAL_GBS, 4),
                      "bytes_per_launch": rf_bytes,
                      "bytes_note": "every launch reads its resident experts' blocks from HBM and writes its missed "
                                    "experts' blocks to HBM: k payloads per launch; traffic is an all-resident "
@@ -424,7 +428,8 @@ def resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, s
         mf.mf_destroy(ctx)
     us = 1e3 * ms / n
     gbs = bytes_per_launch / (us * 1e-6) / 1e9
-    return {"achieved": round(gbs, 1), "frac": round(gbs / hbm, 4), "us_per_launch": round(us, 3), "launches": n,
+    return {"achieved": round(gbs, 1), "frac": round(gbs / hbm, 4), "frac_of_nominal": round(gbs / HBM_NOMINAL_GBS, 4),
+            "us_per_launch": round(us, 3), "launches": n,
             "misses_in_timed_replays": st["misses"],
             "how": "same calls, 100 % cache warmed by two passes (every launch all-resident), L2 flushed per replay",
             "read_floor": read_floor(torch, device, stream, flush, bytes_per_launch, hbm)}
