@@ -376,6 +376,13 @@ def run_mawforge(args):
         runs = [cpu_baseline(args.cpu_tokens, args.cache_pct) for _ in range(args.cpu_passes)]
         line["cpu_baseline"] = dict(runs[0], value=round(statistics.mean(r["value"] for r in runs), 4),
                                     sample=runs[0]["sample"] + f", {args.cpu_passes} passes from a cold cache")
+        others = {}  # the oracle beside the other measured workloads (bounded samples)
+        for name, fn in (("prefill", cpu_baseline_prefill), ("batch64", cpu_baseline_batch64)):
+            try:
+                others[name] = fn()
+            except Exception as e:
+                others[name] = {"error": f"{type(e).__name__}: {e}"}
+        line["cpu_baseline"]["other_workloads"] = others
     if rank == 0:
         print(json.dumps(line))
     if ws > 1:
@@ -805,6 +812,51 @@ def cpu_baseline(n_tokens: int, cache_pct: float = 35.0) -> dict:
             "slots_per_layer": slots,
             "sample": f"first {n_tokens} tokens of the same sequence (256 = the whole step), all {L} layers "
                       f"(router + LRU with {slots} slots + fp64 layer)"}
+
+
+def cpu_baseline_prefill(n_tokens: int = 8, cache_pct: float = 15.0) -> dict:
+    """The CPU oracle on the first tokens of the prefill measurement's 4096-token call (layer 0 of
+    the 48-layer Q4_0 workload, the same inputs): the fp64 layer with its routing, and the call's
+    cache step; tokens/s of one layer, like the GPU's prefill rate."""
+    import oracle
+    import synth
+    cfg = synth.CONFIGS["l48e128q4"]
+    H, E, k, I, q, T = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype, cfg.prefill
+    route = cfg.route_classes[0]
+    x = synth.activations(0, 0, 0, 0, n_tokens, H)
+    b = synth.plant_bias(synth.routes(0, 0, 0, E, k, T, route.zipf_s, route.reuse)[:n_tokens], E)
+    wr = synth.router_weights(cfg.model_seed, 0, E, H)
+    pays = {e: synth.payload(cfg.model_seed, 0, e, H, I, q) for e in set(b.nonzero()[1].tolist())}
+    lru = oracle.LRU(E, max(k, int(np.floor(cache_pct * E / 100 + 1e-9))), synth.payload_bytes(H, I, q))
+    t0 = time.perf_counter()
+    _, idx, _ = oracle.layer([pays.get(e) for e in range(E)], q, H, I, k, wr, b, x)
+    lru.step(idx)
+    dt = time.perf_counter() - t0
+    return {"value": round(n_tokens / dt, 4), "unit": "tokens/s (one layer)", "kind": "oracle",
+            "sample": f"the first {n_tokens} tokens of the 4096-token prefill call, layer 0 of l48e128q4"}
+
+
+def cpu_baseline_batch64(n_streams: int = 8, cache_pct: float = 15.0) -> dict:
+    """The CPU oracle on the first streams of the 64-stream measurement's first call (layer 0 of
+    the 30-layer workload, the same inputs): the fp64 layer with its routing and the cache step;
+    tokens/s of one layer, like the GPU's 64-stream rate."""
+    import oracle
+    import synth
+    cfg = synth.CONFIGS["l30e128b64"]
+    H, E, k, I, q = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    klass = cfg.route_classes[0]
+    routes = np.stack([synth.routes(0, 0, st, E, k, 1, klass.zipf_s, klass.reuse)[0] for st in range(n_streams)])
+    x = np.concatenate([synth.activations(0, 0, st, 0, 1, H) for st in range(n_streams)])
+    b = synth.plant_bias(routes, E)
+    wr = synth.router_weights(cfg.model_seed, 0, E, H)
+    pays = {e: synth.payload(cfg.model_seed, 0, e, H, I, q) for e in set(routes.reshape(-1).tolist())}
+    lru = oracle.LRU(E, max(k, int(np.floor(cache_pct * E / 100 + 1e-9))), synth.payload_bytes(H, I, q))
+    t0 = time.perf_counter()
+    _, idx, _ = oracle.layer([pays.get(e) for e in range(E)], q, H, I, k, wr, b, x)
+    lru.step(idx)
+    dt = time.perf_counter() - t0
+    return {"value": round(n_streams / dt, 4), "unit": "tokens/s (one layer)", "kind": "oracle",
+            "sample": f"the first {n_streams} of the 64 streams of the first call, layer 0 of l30e128b64"}
 
 
 def run_reference(args):

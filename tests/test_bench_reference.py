@@ -43,3 +43,12 @@ def test_cpu_baseline_cache_matches_the_planner():
         r = bench.cpu_baseline(1, pct)
         assert r["slots_per_layer"] == plan.slots_per_layer, pct
         assert r["value"] > 0 and r["kind"] == "oracle"
+
+
+def test_oracle_samples_of_the_other_workloads():
+    """The CPU-baseline leg also times the oracle on bounded samples of the prefill and 64-stream
+    workloads (one layer each), beside the GPU's rates for them."""
+    for fn in (bench.cpu_baseline_prefill, bench.cpu_baseline_batch64):
+        r = fn(2)
+        assert r["kind"] == "oracle" and r["value"] > 0 and r["unit"] == "tokens/s (one layer)"
+        assert "first 2" in r["sample"]
