@@ -353,7 +353,7 @@ def run_mawforge(args):
     line["copy"].update({"h2d_gbs_measured": round(h2d, 1),
                          "link_ms_per_step_at_h2d": round(link_ms, 3),
                          "link_share_of_step": round(link_ms / ms, 4),
-                         "h2d_how": "pinned host -> device cudaMemcpyAsync of 1 GiB, best of 3, this run"})
+                         "h2d_how": "pinned host -> device cudaMemcpyAsync of 1 GiB, best of 10, this run"})
     if n_ff and not args.no_resident and rank == 0:
         line["roofline"]["resident"] = resident_measurement(torch, mf, synth, device, x, bias, wr, stream, flush,
                                                             args.steps, rf_bytes, hbm)
@@ -621,7 +621,7 @@ def spec_measurement(torch, mf, synth, device, x, bias, wr, stream, flush, cache
                              "speculative": round(N_TOKENS / (msv * 1e-3), 1)}}
 
 
-def h2d_bandwidth(torch, device, stream, nbytes: int = 1 << 30, reps: int = 3) -> float:
+def h2d_bandwidth(torch, device, stream, nbytes: int = 1 << 30, reps: int = 10) -> float:
     """GB/s of one pinned host -> device copy engine transfer (the CPU-GPU link's rate for a
     plain copy), best of `reps`."""
     src = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
