@@ -1,7 +1,7 @@
 """bench.py's reference arm on CPU: it times the CPU oracle on a bounded sample of the headline
 workload and prints one JSON line with the same metric, unit, direction and workload as the
 GPU arm, a cpu_baseline object describing the run and an end-to-end object with no copies.
-Two tokens of the four-layer sequence keep it to seconds."""
+Two tokens through four of the 48 layers keep it to seconds."""
 import argparse
 import json
 
@@ -22,7 +22,8 @@ def test_reference_arm_json_line(monkeypatch, capsys):
     assert line["unit"] == "tokens/s" and line["higher_is_better"] is True
     assert line["n_gpus"] == 1 and line["steps"] == 1 and line["warmup"] == 0
     assert line["value"] > 0
-    assert abs(line["ms_per_step"] - 1e3 * 2 / line["value"]) <= 1e-3 * line["ms_per_step"] + 1e-3
+    # value = layer-tokens / 48 per second: 2 tokens x 4 layers per step
+    assert abs(line["ms_per_step"] - 1e3 * (2 * 4 / bench.N_LAYERS) / line["value"]) <= 1e-3 * line["ms_per_step"] + 1e-3
     assert line["config"]["workload"] == bench.workload_name(35.0)
     cb = line["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["unit"] == line["unit"]
@@ -40,7 +41,7 @@ def test_cpu_baseline_cache_matches_the_planner():
     model = mf.Model(cfg.n_layers, cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype)
     for pct in (35.0, 15.0, 1.0):
         plan = mf.mf_plan(model, mf.PlanReq(pct, 1 << 62, 0, 0, 1, 0))
-        r = bench.cpu_baseline(1, pct)
+        r = bench.cpu_baseline(1, pct, 1)
         assert r["slots_per_layer"] == plan.slots_per_layer, pct
         assert r["value"] > 0 and r["kind"] == "oracle"
 
