@@ -234,10 +234,28 @@ int mf_timing(mf_ctx_t* ctx, unsigned class_mask);
 int mf_timing_read(mf_ctx_t* ctx, double* ms, int64_t* launches);
 
 /* Synchronise the device and report whether any kernel of this context gave up a bounded
- * wait since the last check (MF_E_TIMEOUT; results of that call are then unreliable).
- * Kernels never spin without a limit: a pipeline stage that is not filled or released
- * within the limit makes the kernel record the failure and return. */
+ * wait since the last check (MF_E_TIMEOUT), clearing the record.  Kernels never spin without a
+ * limit: a pipeline stage that is not filled or released, or a block whose partner blocks do not
+ * publish their part, within the time limit (mf_wait_limit) makes the kernel record the failure
+ * and return.  After MF_E_TIMEOUT the outputs of the calls since the last check are unreliable,
+ * and so may be the contents of slots materialised by them: call mf_reset before relying on the
+ * cache again.  The context itself stays usable. */
 int mf_check(mf_ctx_t* ctx);
+
+/* Time limit, in seconds (1e-6 .. 60), of every bounded wait inside this context's kernels
+ * (default 1 s): a wait that has not completed after that long gives up as described under
+ * mf_check.  MF_E_INVAL outside the range.  Host only; applies to calls issued afterwards
+ * (calls already captured into a CUDA graph keep the limit they were captured with). */
+int mf_wait_limit(mf_ctx_t* ctx, double seconds);
+
+/* Test hold for the failure path (no counterpart in the paper).  hold = 1: the producer warp of
+ * the one-token expert FFN kernel issues none of its HBM copies, so the stages its consumers wait
+ * for are never filled: their bounded waits run out after the wait limit, the kernel records the
+ * failure and returns with nothing in flight, and mf_check reports MF_E_TIMEOUT.  Nothing faults
+ * or hangs.  Calls whose experts all hit move no other bytes, so the cache stays consistent;
+ * hold = 0 (the default) restores normal operation.  MF_E_INVAL for other values.  Host only;
+ * applies to calls issued afterwards. */
+int mf_test_hold(mf_ctx_t* ctx, int hold);
 
 /* One-token expert FFN with no allocation at all (the paper has no counterpart: it is a
  * convenience of this library).  Callers that cannot allocate device memory — code running
@@ -265,11 +283,20 @@ int mf_check(mf_ctx_t* ctx);
  *            aligned; y device float [hidden] output
  * Stream-ordered on `stream`; returns after enqueueing.  The first call on each device sets up
  * that device (it reads the array's device address and writes its constant tables): make that
- * first call before any stream capture.  All calls on a device share the array, so calls whose
- * kernels overlap on the GPU (other streams, other host threads) race on it: serialise them.
- * Nothing in the array needs clearing between calls; h is fully rewritten by each call. */
+ * first call before any stream capture; host threads that make their first call at the same time
+ * take turns.  All calls on a device share the array, so calls whose kernels overlap on the GPU
+ * (other streams, other host threads) race on it: serialise them.  Nothing in the array needs
+ * clearing between calls; h is fully rewritten by each call.  A bounded wait that gives up is
+ * reported by mf_expert_ffn_noalloc_check. */
 int mf_expert_ffn_noalloc(const mf_model_t* model, const void* experts, const float* g, const float* x,
                           float* y, void* stream);
+
+/* Failure report of mf_expert_ffn_noalloc on the current device (its kernels' bounded waits give
+ * up after 1 s and record that in the same static array): synchronises the device and returns
+ * MF_E_TIMEOUT if a wait gave up since the last check, clearing the record, else MF_OK (also
+ * when no call has run on the device).  Allocates nothing; MF_E_CUDA if the device cannot be
+ * read. */
+int mf_expert_ffn_noalloc_check(void);
 
 /* Release everything the context owns (synchronises its streams first). NULL is a no-op. */
 void mf_destroy(mf_ctx_t* ctx);

@@ -17,7 +17,8 @@ import os
 __all__ = [
     "MFError", "Model", "PlanReq", "Plan", "Stats", "TunePoint", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
     "mf_payload_bytes", "mf_plan", "mf_tune_cache", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
-    "mf_moe_forward_host", "mf_prefill_threshold", "mf_access_order", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_expert_ffn_noalloc", "mf_destroy",
+    "mf_moe_forward_host", "mf_prefill_threshold", "mf_access_order", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_wait_limit", "mf_test_hold", "mf_expert_ffn_noalloc",
+    "mf_expert_ffn_noalloc_check", "mf_destroy",
     "mf_strerror", "mf_last_cuda_error",
 ]
 
@@ -90,7 +91,10 @@ _sig = {
     "mf_timing": (_i32, [_vp, ctypes.c_uint]),
     "mf_timing_read": (_i32, [_vp, _vp, _vp]),
     "mf_check": (_i32, [_vp]),
+    "mf_wait_limit": (_i32, [_vp, ctypes.c_double]),
+    "mf_test_hold": (_i32, [_vp, _i32]),
     "mf_expert_ffn_noalloc": (_i32, [ctypes.POINTER(Model), _vp, _vp, _vp, _vp, _vp]),
+    "mf_expert_ffn_noalloc_check": (_i32, []),
     "mf_destroy": (None, [_vp]),
     "mf_strerror": (ctypes.c_char_p, [_i32]),
     "mf_last_cuda_error": (ctypes.c_char_p, []),
@@ -270,6 +274,25 @@ def mf_check(ctx: int) -> int:
     rc = _lib.mf_check(ctx)
     if rc not in (MF_OK, MF_E_TIMEOUT):
         _check(rc, "mf_check")
+    return rc
+
+
+def mf_wait_limit(ctx: int, seconds: float) -> None:
+    """Time limit of every bounded wait inside the context's kernels."""
+    _check(_lib.mf_wait_limit(ctx, float(seconds)), "mf_wait_limit")
+
+
+def mf_test_hold(ctx: int, hold: int) -> None:
+    """Test hold of the failure path: 1 = the one-token FFN's producer issues no copies."""
+    _check(_lib.mf_test_hold(ctx, int(hold)), "mf_test_hold")
+
+
+def mf_expert_ffn_noalloc_check() -> int:
+    """0, or MF_E_TIMEOUT if a no-allocation call on the current device gave up a bounded wait since
+    the last check (returned, not raised)."""
+    rc = _lib.mf_expert_ffn_noalloc_check()
+    if rc not in (MF_OK, MF_E_TIMEOUT):
+        _check(rc, "mf_expert_ffn_noalloc_check")
     return rc
 
 

@@ -117,7 +117,7 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.miss_list = c.take<int32_t>(E + S);
   o.h = c.take<float>((uint64_t)Tm * k * I);
   o.part = c.take<float>(Tm > 1 ? (uint64_t)Tm * k * H : 1);
-  o.work = c.take<unsigned>(4);
+  o.work = c.take<uint64_t>(16);  // the fused FFN's grid arrival counter, alone on its 128-byte line
   o.err = c.take<unsigned>(1);
   o.tb_off = c.take<int32_t>(E + 1);
   o.sx = c.take<float>((uint64_t)Tm * H);
@@ -328,6 +328,8 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.T_max = Tm;
   d.order = MF_ORDER_FIRST_OCCURRENCE;
   d.lay = make_layout(*m);
+  d.wait_ns = kDefaultWaitNs;
+  d.hold = 0;
 
   int rc = MF_OK;
   cudaError_t e;
@@ -390,7 +392,7 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   d.miss_list = reinterpret_cast<int32_t*>(base + so.miss_list);
   d.h = reinterpret_cast<float*>(base + so.h);
   d.part = reinterpret_cast<float*>(base + so.part);
-  d.work = reinterpret_cast<unsigned*>(base + so.work);
+  d.work = reinterpret_cast<unsigned long long*>(base + so.work);
   d.stage = Tm > 1 ? base + so.stage : nullptr;
   d.err = reinterpret_cast<unsigned*>(base + so.err);
   d.tb_off = reinterpret_cast<int32_t*>(base + so.tb_off);
@@ -750,6 +752,18 @@ int mf_timing_read(mf_ctx_t* c, double* ms, int64_t* launches) {
     ms[i] = acc;
     launches[i] = c->timer_n[i];
   }
+  return MF_OK;
+}
+
+int mf_wait_limit(mf_ctx_t* c, double seconds) {
+  if (!c || !(seconds >= 1e-6 && seconds <= 60.0)) return MF_E_INVAL;
+  c->d.wait_ns = (uint64_t)(seconds * 1e9);
+  return MF_OK;
+}
+
+int mf_test_hold(mf_ctx_t* c, int hold) {
+  if (!c || (hold != 0 && hold != 1)) return MF_E_INVAL;
+  c->d.hold = hold;
   return MF_OK;
 }
 

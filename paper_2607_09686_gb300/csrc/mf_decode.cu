@@ -76,13 +76,36 @@ size_t smem_bytes(const PipeCfg& c) {
   return (size_t)c.NS * c.stage_bytes + 2 * kMaxStages * sizeof(uint64_t) + part_bytes(c.max_mine) + c.vq_bytes;
 }
 
-// The consumers split `n` vectors of kW values into int8 pieces, one vector per thread, into
-// shared memory, then wait for each other (the producer keeps streaming meanwhile).
+// The consumers split `n` groups of kW values into int8 pieces in shared memory (XQ).  Groups
+// [r * per, (r + 1) * per) form one vector r (x, or one expert's h), split as if scaled by one
+// power of two: each group is split with its own exponent, the vector's exponent e_r (the largest,
+// a shared-memory atomic max) goes to s_exp[r], and each group's s is then rescaled to it.
+// s_max[r] must hold kNoExp on entry; n <= 4 * 512.  The producer keeps streaming meanwhile.
 template <int QT, bool kCoherent = false>
-__device__ __forceinline__ void split_vectors(const float* __restrict__ src, int n, XQ<QT>* dst) {
-  for (int i = threadIdx.x; i < n; i += kConsumers * 32)
-    dst[i] = quant_vec<QT, kCoherent>(src + (size_t)i * Vec<QT>::kW);
-  named_bar_sync(1, kConsumers * 32);
+__device__ __forceinline__ void split_vectors(const float* __restrict__ src, int n, int per, XQ<QT>* dst,
+                                              int* s_max, int* s_exp) {
+  constexpr int kW = Vec<QT>::kW;
+  const int nt = kConsumers * 32, i0 = (int)threadIdx.x;
+  int eg[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = i0 + q * nt;
+    if (i < n) {
+      float v[kW];
+      load_group<QT, kCoherent>(src + (size_t)i * kW, v);
+      eg[q] = group_exponent(group_absmax<QT>(v));
+      dst[i] = quant_vals<QT>(v, eg[q] == kNoExp ? 0 : -eg[q]);
+      atomicMax(&s_max[i / per], eg[q]);
+    }
+  }
+  named_bar_sync(1, nt);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    const int i = i0 + q * nt;
+    if (i < n) rescale_group<QT>(dst[i], eg[q], vector_exponent(s_max[i / per]));
+  }
+  for (int r = i0; r * per < n; r += nt) s_exp[r] = vector_exponent(s_max[r]);
+  named_bar_sync(1, nt);
 }
 
 // Items of this block: blockIdx.x, blockIdx.x + gridDim.x, ...  Producer and consumers both
@@ -116,10 +139,10 @@ __device__ __forceinline__ void init_barriers(const PipeCfg& c, const Smem& sm) 
 
 // Producer epilogue: wait (bounded) for the last use of every stage, so that no copy is in
 // flight when the block exits even if the consumers stopped early.
-__device__ __forceinline__ void drain(const PipeCfg& c, const Smem& sm, int mine, unsigned* err) {
+__device__ __forceinline__ void drain(const PipeCfg& c, const Smem& sm, int mine, unsigned* err, uint64_t limit_ns) {
   for (int s = 0; s < c.NS && s < mine; ++s) {
     const int uses = (mine - 1 - s) / c.NS + 1;  // iterations it < mine with it % NS == s
-    if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u)) atomicExch(err, 2u);
+    if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u, limit_ns)) atomicExch(err, 2u);
   }
 }
 
@@ -130,6 +153,8 @@ template <int QT, int VPL>
 __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, const float* __restrict__ x, PipeCfg c) {
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ const uint8_t* s_base[kMaxTopK];  // slot of each routed expert
+  __shared__ int s_xmax;
+  __shared__ int s_xexp;
   const Smem sm = carve(smem, c);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qrow = d.lay.qrow_gu;
@@ -138,6 +163,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, c
   const int mine = items_of_block(c.n_items);
   if (threadIdx.x < d.k)
     s_base[threadIdx.x] = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
+  if (threadIdx.x == 0) s_xmax = kNoExp;
   init_barriers(c, sm);
 
   if (warp == kConsumers) {
@@ -146,7 +172,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, c
       int u = (int)blockIdx.x / nrb, rb = (int)blockIdx.x % nrb;
       Ring ring;
       for (int it = 0; it < mine; ++it) {
-        if (it >= c.NS && !mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u)) {
+        if (it >= c.NS && !mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u, d.wait_ns)) {
           atomicExch(d.err, 1u);
           break;
         }
@@ -160,23 +186,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, c
           ++u;
         }
       }
-      drain(c, sm, mine, d.err);
+      drain(c, sm, mine, d.err, d.wait_ns);
     }
   } else {
     const int ten = warp / (R * cs), row = (warp / cs) % R, col = warp % cs;
     const int nv = (qrow / 16) / cs;  // vectors in this warp's column range
     const int v0 = col * nv;
     const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-    split_vectors<QT>(x, c.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq));
+    split_vectors<QT>(x, c.n_vec, c.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq), &s_xmax, &s_xexp);
     XQ<QT> xr[VPL];
 #pragma unroll
     for (int i = 0; i < VPL; ++i) {
       const int v = lane + 32 * i;
       if (v < nv) xr[i] = xq[v0 + v];
     }
+    const int ex = s_xexp;
     Ring ring;
     for (int it = 0; it < mine; ++it) {
-      if (!mbar_wait(&sm.full[ring.s], ring.phase)) {
+      if (!mbar_wait(&sm.full[ring.s], ring.phase, d.wait_ns)) {
         if (lane == 0) atomicExch(d.err, 3u);
         break;
       }
@@ -199,7 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, c
       ring.next(c.NS);
     }
     // all partial results of the block are in shared memory: SwiGLU over (item, row), column
-    // ranges added in order
+    // ranges added in order, times 2^ex (x was split scaled by 2^-ex)
     named_bar_sync(1, kConsumers * 32);
     for (int t = threadIdx.x; t < mine * R; t += kConsumers * 32) {
       const int it = t / R, r = t % R;
@@ -209,6 +236,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_gateup_pipe(Dev d, int layer, c
         ag += p[(0 * R + r) * cs + cc];
         au += p[(1 * R + r) * cs + cc];
       }
+      ag = scale2(ag, ex);
+      au = scale2(au, ex);
       const int item = (int)blockIdx.x + it * (int)gridDim.x;
       d.h[(size_t)(item / nrb) * d.I + (item % nrb) * R + r] = ag / (1.0f + expf(-ag)) * au;
     }
@@ -223,6 +252,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ float s_g[kMaxTopK];
   __shared__ const uint8_t* s_base[kMaxTopK];
+  __shared__ int s_hmax[kMaxTopK];
+  __shared__ int s_hexp[kMaxTopK];
   const Smem sm = carve(smem, c);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int k = d.k, R = c.R;
@@ -233,7 +264,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
     s_g[threadIdx.x] = d.g[threadIdx.x];
     s_base[threadIdx.x] = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride + d.lay.d_off;
   }
-  init_barriers(c, sm);  // (its barrier also publishes s_g and s_base)
+  if (threadIdx.x < kMaxTopK) s_hmax[threadIdx.x] = kNoExp;
+  init_barriers(c, sm);  // (its barrier also publishes s_g, s_base and s_hmax)
 
   if (warp == kConsumers) {
     if (lane == 0) {
@@ -242,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
       size_t c0 = (size_t)blockIdx.x * R;
       const size_t c_step = (size_t)gridDim.x * R;
       for (int it = 0; it < mine; ++it) {
-        if (it >= c.NS && !mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u)) {
+        if (it >= c.NS && !mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u, d.wait_ns)) {
           atomicExch(d.err, 1u);
           break;
         }
@@ -253,13 +285,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
         ring.next(c.NS);
         c0 += c_step;
       }
-      drain(c, sm, mine, d.err);
+      drain(c, sm, mine, d.err, d.wait_ns);
     }
   } else {
     const int j = warp / R, rho = warp % R;  // one (expert, row) task per warp: k * R <= 16
     const bool active = j < k;
     const XQ<QT>* hq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-    split_vectors<QT>(d.h, c.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq));  // h of all k experts
+    split_vectors<QT>(d.h, c.n_vec, nvec, reinterpret_cast<XQ<QT>*>(sm.vq), s_hmax, s_hexp);  // h of all k experts
     XQ<QT> hr[VPLD];
     if (active) {
 #pragma unroll
@@ -270,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
     }
     Ring ring;
     for (int it = 0; it < mine; ++it) {
-      if (!mbar_wait(&sm.full[ring.s], ring.phase)) {
+      if (!mbar_wait(&sm.full[ring.s], ring.phase, d.wait_ns)) {
         if (lane == 0) atomicExch(d.err, 4u);
         break;
       }
@@ -293,13 +325,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
       if (lane == 0) mbar_arrive(&sm.empty[ring.s]);
       ring.next(c.NS);
     }
-    // combine the k experts of each output row in rank order
+    // combine the k experts of each output row in rank order (expert j's partial times 2^e_j:
+    // its h was split scaled by 2^-e_j)
     named_bar_sync(1, kConsumers * 32);
     for (int t = threadIdx.x; t < mine * R; t += kConsumers * 32) {
       const int it = t / R, r = t % R;
       const float* p = sm.red + it * kConsumers;
       float acc = 0.f;
-      for (int jj = 0; jj < k; ++jj) acc = fmaf(s_g[jj], p[jj * R + r], acc);
+      for (int jj = 0; jj < k; ++jj) acc = fmaf(s_g[jj], scale2(p[jj * R + r], s_hexp[jj]), acc);
       y[((size_t)blockIdx.x + (size_t)it * gridDim.x) * R + r] = acc;
     }
   }
@@ -307,22 +340,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 }
 
 // ---------------------------------------------------------------- fused gate/up + down, one token
-// Both projections in one persistent cooperative launch, which also materialises the call's
-// missed experts.  The gate/up items are dealt round-robin over the blocks from a list that
-// holds the resident experts' items first, so every block gets an equal share (+-1) of the
-// missed ones.  The producer warp streams the resident items from HBM through ring A; a link
-// warp, from the first cycle, reads the missed items straight from the pinned pack (16-byte
-// loads over the host link) into the stages of a small ring B and writes each through to the
-// expert's new HBM slot, then does the same for the missed experts' down records, so the link
-// transfer overlaps the resident data and all compute.  The consumers take ring A's items, then
-// ring B's.  A block's down work is a contiguous
-// range of rpc output rows: its item j is expert j's rpc down records, one bulk copy into a buffer
-// of its own.  The producer requests those k copies right after the first gate/up items (the down
-// weights do not depend on h), then streams the rest of the gate/up items through the ring, so the
-// whole call's weights are in flight from the start.  The consumers form h = silu(gate) * up for
-// their gate/up items, publish it, meet every other block at a grid-wide arrival counter (bounded
-// wait), and then take the down items with the k experts' h.  The counter never resets: each launch adds one
-// arrival per block, and a block waits for the multiple of gridDim.x that completes its launch.
+// Both projections in one persistent launch, which also materialises the call's missed
+// experts.  The gate/up items are dealt round-robin over the blocks from a list that holds the
+// resident experts' items first, so every block gets an equal share (+-1) of the missed ones.
+// The producer warp streams the resident items from HBM through ring A; a link warp, from the
+// first cycle, reads the missed items straight from the pinned pack (16-byte loads over the host
+// link) into the stages of a small ring B and writes each through to the expert's new HBM slot,
+// then does the same for the missed experts' down records, so the link transfer overlaps the
+// resident data and all compute.  The consumers take ring A's items, then ring B's.  A block's
+// down work is a contiguous range of rpc output rows: its item j is expert j's rpc down records,
+// one bulk copy into a buffer of its own.  The producer requests those k copies right after the
+// first gate/up items (the down weights do not depend on h), then streams the rest of the gate/up
+// items through the ring, so the whole call's weights are in flight from the start.  The
+// consumers form h = silu(gate) * up for their gate/up items, publish it, meet every other block
+// at a grid-wide arrival counter (bounded wait), and then take the down items with the k experts'
+// h.  The counter never resets: each launch adds one arrival per block, and a block waits for the
+// multiple of gridDim.x that completes its launch.
+//
 // Missed experts' bytes, by the whole warp: host_pull issues `bytes` (a multiple of 16) from the
 // pinned pack into shared memory as 16-byte cp.async pieces (every piece in flight at once; the
 // caller commits and waits); once they have landed, slot_write_through makes the warp's
@@ -363,19 +397,15 @@ struct FusedCfg {
   // shared memory: [NS gate/up stages | k down buffers | full | empty | full_d | red | vq]
   size_t off_dn, off_bar, off_red, off_vq, total;
 };
+constexpr int kFusedBars = 2 * kMaxStages + kMaxTopK;
 
 // The arrival is a release (the block's h, written before it and published to this thread by the
-// block barrier, becomes visible with it); the polling loads acquire.
-__device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, unsigned* err) {
+// block barrier, becomes visible with it); the polling loads acquire.  Bounded in time.
+__device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, unsigned* err, uint64_t limit_ns) {
   unsigned long long old;
   asm volatile("atom.add.release.gpu.global.u64 %0, [%1], 1;" : "=l"(old) : "l"(arrive) : "memory");
   const unsigned long long target = (old / gridDim.x + 1) * gridDim.x;
-  for (uint32_t i = 0; i < (1u << 22); ++i) {
-    unsigned long long v;
-    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(arrive) : "memory");
-    if (v >= target) return true;
-    if (i >= 64) __nanosleep(32);
-  }
+  if (counter_wait(arrive, target, limit_ns)) return true;
   atomicExch(err, 5u);
   return false;
 }
@@ -383,6 +413,7 @@ __device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, uns
 template <int QT, int VPL, int VPLD>
 __global__ void __launch_bounds__(kThreadsF, 1)
     k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, float* __restrict__ y, FusedCfg f) {
+  constexpr int kW = Vec<QT>::kW;
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ uint8_t* s_gu[kMaxTopK];  // each expert's HBM slot: gate/up region, down region
   __shared__ uint8_t* s_dn[kMaxTopK];
@@ -392,6 +423,8 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   __shared__ int s_gord[kMaxItemsF];  // the block's gate/up items: resident experts' first
   __shared__ int s_ord[kMaxTopK];     // ranks: resident experts', then missed experts'
   __shared__ int s_nres, s_nb;        // how many of them are resident; ring B's stages
+  __shared__ int s_xmax, s_xexp;      // exponent of x's largest magnitude (split scale)
+  __shared__ int s_hmax[kMaxTopK], s_hexp[kMaxTopK];  // the same for each expert's h
   const PipeCfg& cg = f.g;
   Smem sm;
   sm.stage0 = smem;
@@ -406,6 +439,21 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   const int mine_g = items_of_block(cg.n_items);
   const int r0 = (int)blockIdx.x * f.rpc, nrows = max(0, min(d.H - r0, f.rpc));  // this block's down rows
   const int mine_d = nrows > 0 ? k : 0;
+  // prologue: this block's shared memory only (with a programmatic launch it overlaps the router)
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < f.NS; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], kConsumers);
+    }
+    for (int j = 0; j < k; ++j) mbar_init(&full_d[j], 1);
+    mbar_fence_init();
+    s_xmax = kNoExp;
+  }
+  if (threadIdx.x < kMaxTopK) s_hmax[threadIdx.x] = kNoExp;
+  pdl_wait();  // the router's outputs (and the caller's x) are complete and visible
+  float xv[kW];  // consumer thread i < n_vec: group i of x, requested while the block sets up
+  const bool x_mine = warp < kConsumers && (int)threadIdx.x < cg.n_vec;
+  if (x_mine) load_group<QT>(x + (size_t)threadIdx.x * kW, xv);
   if (threadIdx.x < k) {  // one token: access u = rank j
     uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
     s_gu[threadIdx.x] = slot;
@@ -433,18 +481,13 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     }
     s_nres = nres;
     s_nb = n_res_e < k ? 2 : 0;  // ring B only when the call has a missed expert (NS >= 4)
-    for (int s = 0; s < f.NS; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], kConsumers);
-    }
-    for (int j = 0; j < k; ++j) mbar_init(&full_d[j], 1);
-    mbar_fence_init();
   }
   __syncthreads();
 
   const int nres = s_nres, NB = s_nb, NA = f.NS - NB;  // ring A: stages [0, NA); ring B: [NA, NS)
   if (warp == kConsumers) {
-    // ---- producer warp: lane 0 streams the resident experts' items and down records
+    // ---- producer warp: lane 0 streams the resident experts' items and down records (none while
+    // the context's test hold is set)
     Ring ring;
     int it = 0;
     bool ok = true;
@@ -452,8 +495,9 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
     const uint32_t dbytes = (uint32_t)nrows * d.lay.rs_d;
     const size_t doff = (size_t)r0 * d.lay.rs_d;
+    const int n_issue = d.hold ? 0 : nres;
     // the resident experts' down records go after the first two gate/up items
-    const int first = min(nres, min(2, NA));
+    const int first = min(n_issue, min(2, NA));
     const uint64_t pol = l2_evict_first();  // read once per call: keep L2 for what is reused
     bool d_issued = false;
     auto issue_down_hits = [&]() {
@@ -466,25 +510,25 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       d_issued = true;
     };
     if (lane == 0) {
-      for (int t = 0; t < nres; ++t, ++it) {
+      for (int t = 0; t < n_issue; ++t, ++it) {
         if (t == first) issue_down_hits();
-        if (it >= NA && !(ok = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u))) break;
+        if (it >= NA && !(ok = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u, d.wait_ns))) break;
         const int item = s_gord[t], u = item / nrb, rb = item % nrb;
         uint64_t* bar = &sm.full[ring.s];
         mbar_arrive_tx(bar, bytes);
         bulk_g2s_hint(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar, pol);
         ring.next(NA);
       }
-      if (ok && !d_issued) issue_down_hits();
+      if (ok && !d_issued && !d.hold) issue_down_hits();
       if (!ok) atomicExch(d.err, 1u);
       // no copy may be in flight when the block exits: wait for the last use of every stage
       for (int s = 0; s < NA && s < it; ++s) {
         const int uses = (it - 1 - s) / NA + 1;
-        if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u)) atomicExch(d.err, 2u);
+        if (!mbar_wait(&sm.full[s], (uint32_t)(uses - 1) & 1u, d.wait_ns)) atomicExch(d.err, 2u);
       }
       if (d_issued)
         for (int j = 0; j < mine_d; ++j)
-          if (!s_miss[j] && !mbar_wait(&full_d[j], 0)) atomicExch(d.err, 2u);
+          if (!s_miss[j] && !mbar_wait(&full_d[j], 0, d.wait_ns)) atomicExch(d.err, 2u);
     }
   } else if (warp == kConsumers + 1) {
     // ---- link warp: the missed experts' items through ring B (both stages in flight at once),
@@ -515,7 +559,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       if (issued < n_li) {  // refill the stage once the consumers are done with item t
         int w = 1;
         if (lane == 0) {
-          w = mbar_wait(&sm.empty[NA + s], (uint32_t)(t / NB) & 1u);
+          w = mbar_wait(&sm.empty[NA + s], (uint32_t)(t / NB) & 1u, d.wait_ns);
           slot_writes_read();  // and its write-through has read it
         }
         if (!__shfl_sync(0xffffffffu, w, 0)) {
@@ -526,6 +570,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
         ++issued;
       }
     }
+    if (!ok) asm volatile("cp.async.wait_all;" ::: "memory");  // nothing of ours in flight at exit
     if (ok) {
       bool any = false;
       for (int j = 0; j < mine_d; ++j)
@@ -557,7 +602,18 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       const int nv = (d.lay.qrow_gu / 16) / cs;
       const int v0 = col * nv;
       const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-      split_vectors<QT>(x, cg.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq));
+      {  // x split into int8 pieces, scaled by the power of two of its largest magnitude
+        XQ<QT>* dst = reinterpret_cast<XQ<QT>*>(sm.vq);
+        const int eg = x_mine ? group_exponent(group_absmax<QT>(xv)) : kNoExp;
+        if (x_mine) {
+          dst[threadIdx.x] = quant_vals<QT>(xv, eg == kNoExp ? 0 : -eg);
+          atomicMax(&s_xmax, eg);
+        }
+        named_bar_sync(1, kConsumers * 32);
+        if (x_mine) rescale_group<QT>(dst[threadIdx.x], eg, vector_exponent(s_xmax));
+        if (threadIdx.x == 0) s_xexp = vector_exponent(s_xmax);
+        named_bar_sync(1, kConsumers * 32);
+      }
       XQ<QT> xr[VPL];
 #pragma unroll
       for (int i = 0; i < VPL; ++i) {
@@ -567,7 +623,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       for (int it = 0; it < mine_g; ++it) {
         const bool link = it >= nres;  // a missed expert's item: ring B
         const int bi = link ? NA + ring_b.s : ring.s;
-        if (!(ok = mbar_wait(&sm.full[bi], link ? ring_b.phase : ring.phase))) break;
+        if (!(ok = mbar_wait(&sm.full[bi], link ? ring_b.phase : ring.phase, d.wait_ns))) break;
         const unsigned char* rec = sm.stage0 + (size_t)bi * f.stage_bytes + row * rs;
         const unsigned char* q = rec + ten * d.lay.o_up + 16 * v0;
         const __half* sc = reinterpret_cast<const __half*>(rec + (ten ? d.lay.o_us : d.lay.o_gs));
@@ -588,7 +644,10 @@ __global__ void __launch_bounds__(kThreadsF, 1)
         else
           ring.next(NA);
       }
+      // SwiGLU of the block's items (column ranges added in order, times 2^ex: x was split
+      // scaled by 2^-ex)
       named_bar_sync(1, kConsumers * 32);
+      const int ex = s_xexp;
       for (int t = threadIdx.x; t < mine_g * R; t += kConsumers * 32) {
         const int it = t / R, r = t % R;
         const float* p = sm.red + it * kConsumers;
@@ -597,13 +656,16 @@ __global__ void __launch_bounds__(kThreadsF, 1)
           ag += p[(0 * R + r) * cs + cc];
           au += p[(1 * R + r) * cs + cc];
         }
+        ag = scale2(ag, ex);
+        au = scale2(au, ex);
         const int item = s_gord[it];
         d.h[(size_t)(item / nrb) * d.I + (item % nrb) * R + r] = ag / (1.0f + expf(-ag)) * au;
       }
       named_bar_sync(1, kConsumers * 32);  // the block's h written
     }
+    if (!ok && lane == 0) atomicExch(d.err, 3u);
     // ---- every block's h published (one arrival per block, always, so launches stay aligned)
-    if (threadIdx.x == 0 && !grid_arrive_wait(reinterpret_cast<unsigned long long*>(d.work), d.err)) ok = false;
+    if (threadIdx.x == 0 && !grid_arrive_wait(d.work, d.err, d.wait_ns)) ok = false;
     named_bar_sync(1, kConsumers * 32);
     // ---- down: warp w holds expert j = w / (16 / k)'s h in registers for the whole phase and
     // takes rows sub, sub + 16 / k, ... of that expert's item (sub = w % (16 / k))
@@ -611,7 +673,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       const int nvec = d.lay.qrow_d / 16;
       const uint32_t rs = d.lay.rs_d;
       const XQ<QT>* hq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-      split_vectors<QT, true>(d.h, f.n_hvec, reinterpret_cast<XQ<QT>*>(sm.vq));  // written by other blocks
+      split_vectors<QT, true>(d.h, f.n_hvec, nvec, reinterpret_cast<XQ<QT>*>(sm.vq), s_hmax, s_hexp);  // other blocks wrote h
       float* red = sm.red + cg.max_mine * kConsumers;  // [k][rpc]
       const int wpe = kConsumers / k, j = warp / wpe, sub = warp % wpe;
       if (j < mine_d && ok) {
@@ -621,7 +683,8 @@ __global__ void __launch_bounds__(kThreadsF, 1)
           const int v = lane + 32 * i;
           if (v < nvec) hr[i] = hq[j * nvec + v];
         }
-        if ((ok = mbar_wait(&full_d[j], 0))) {
+        const int e = s_hexp[j];
+        if ((ok = mbar_wait(&full_d[j], 0, d.wait_ns))) {
           const unsigned char* st = dbuf + (size_t)j * f.dn_bytes;
           // four rows at a time: independent dot products and interleaved reductions
           for (int row0 = sub; row0 < nrows; row0 += 4 * wpe) {
@@ -649,7 +712,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
             if (lane == 0)
 #pragma unroll
               for (int rr = 0; rr < 4; ++rr)
-                if (row0 + rr * wpe < nrows) red[j * f.rpc + row0 + rr * wpe] = acc[rr];
+                if (row0 + rr * wpe < nrows) red[j * f.rpc + row0 + rr * wpe] = scale2(acc[rr], e);
           }
         }
       }
@@ -780,14 +843,14 @@ FusedCfg fused_cfg(const Dev& d) {
   f.stage_bytes = f.g.stage_bytes;
   f.red_floats = f.g.max_mine * kConsumers + d.k * f.rpc;
   f.vq_bytes = f.g.vq_bytes > hv_bytes ? f.g.vq_bytes : hv_bytes;
-  const size_t fixed = (size_t)d.k * f.dn_bytes + (2 * kMaxStages + kMaxTopK) * sizeof(uint64_t) +
+  const size_t fixed = (size_t)d.k * f.dn_bytes + kFusedBars * sizeof(uint64_t) +
                        (size_t)f.red_floats * sizeof(float) + f.vq_bytes;
   const size_t budget = kFusedSmem - 1024;  // - the kernel's static shared memory
   const size_t ns = fixed < budget ? (budget - fixed) / f.stage_bytes : 0;
   f.NS = (int)(ns > (size_t)kMaxStages ? kMaxStages : ns);
   f.off_dn = (size_t)f.NS * f.stage_bytes;
   f.off_bar = f.off_dn + (size_t)d.k * f.dn_bytes;
-  f.off_red = f.off_bar + (2 * kMaxStages + kMaxTopK) * sizeof(uint64_t);
+  f.off_red = f.off_bar + kFusedBars * sizeof(uint64_t);
   f.off_vq = f.off_red + (((size_t)f.red_floats * sizeof(float) + 15) & ~(size_t)15);
   f.total = f.off_vq + f.vq_bytes;
   return f;
@@ -795,9 +858,13 @@ FusedCfg fused_cfg(const Dev& d) {
 
 size_t fused_smem(const FusedCfg& f) { return f.total; }
 
+// One block per SM.  The launch is programmatic (it may begin while the router finishes: the
+// kernel's prologue touches only shared memory and it waits for the router before reading
+// anything else); where the driver refuses that, a cooperative launch.  Blocks wait for each
+// other only through bounded waits.
 template <class Kern>
-cudaError_t launch_coop(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x, float* y,
-                        const FusedCfg& f) {
+cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x, float* y,
+                       const FusedCfg& f) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -806,10 +873,19 @@ cudaError_t launch_coop(Kern kern, size_t smem, cudaStream_t s, const Dev& d, in
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeCooperative;  // every block resident: they wait for each other
-  attr[0].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
+  static bool pdl_ok = true;
+  if (pdl_ok) {
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    e = cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
+    if (e == cudaSuccess) return e;
+    cudaGetLastError();
+    pdl_ok = false;
+  }
+  attr[0].id = cudaLaunchAttributeCooperative;  // every block resident: they wait for each other
+  attr[0].val.cooperative = 1;
   return cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
 }
 
@@ -819,7 +895,7 @@ cudaError_t ffn_pipe_q(const Dev& d, int layer, const float* x, float* y, cudaSt
   const size_t smem = fused_smem(f);
   const int vx = vpl_for((d.lay.qrow_gu / 16) / f.g.cs), vh = vpl_for(d.lay.qrow_d / 16);
 #define MF_FF(A, B) \
-  if (vx == A && vh == B) return launch_coop(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, y, f);
+  if (vx == A && vh == B) return launch_ffn(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, y, f);
   MF_FF(1, 1) MF_FF(1, 2) MF_FF(2, 1) MF_FF(2, 2)
   if constexpr (QT == kQ8) {  // Q4_0 takes at most two vectors per lane (decode_pipe_ok)
     MF_FF(1, 3) MF_FF(2, 3) MF_FF(3, 1) MF_FF(3, 2) MF_FF(3, 3) MF_FF(4, 1) MF_FF(4, 2) MF_FF(4, 3)

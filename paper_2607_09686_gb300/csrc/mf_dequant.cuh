@@ -106,6 +106,14 @@ __device__ __forceinline__ float dot_vec(uint4 w, const XV<QT>& x) {
 //   sum_j (c_j - off) v_j ~= s * ((P1 * 127 + P2 - off * (S1 * 127 + S2)) * 127 + P3 - off * S3) / 127^2
 // where S_i = sum_j p_i[j] and off is the code offset (128 for Q8_0's stored q + 128, 8 for Q4_0).
 // Every integer sum is exact (|P1 * 127| < 2^27); fp32 rounds only the final combination.
+//
+// Range: every group of one logical vector (all of x, or one expert's h) is split as if first
+// multiplied by the same power of two 2^-e, e the binary exponent of the vector's largest
+// magnitude, so the largest group maximum lies in [0.5, 1): 127 / max never overflows and s stays
+// a normal number for any finite input, however small or large.  Scaling by a power of two is
+// exact, so the pieces (and every product) are those of the unscaled vector; a result is
+// multiplied back by 2^e once per output row (scale2).  A group whose maximum is below 2^-100 of
+// the vector's is taken as zero (its contribution is below 2^-88 of the row's largest term).
 template <int QT>
 struct XQ {
   static constexpr int kWords = Vec<QT>::kW / 4;  // words of four values: 4 (Q8_0) or 8 (Q4_0)
@@ -114,13 +122,40 @@ struct XQ {
   float sf;     // s / 127^2
 };
 
-// kCoherent: read through L2 only (for vectors other blocks of the same kernel wrote)
+// 2^n as a binary32 value, for -126 <= n <= 127
+__device__ __forceinline__ float pow2i(int n) { return __uint_as_float((uint32_t)(127 + n) << 23); }
+// v * 2^n, exact unless the result leaves the binary32 range (|n| <= 252: two normal factors)
+__device__ __forceinline__ float scale2(float v, int n) {
+  const int a = n / 2;
+  return v * pow2i(a) * pow2i(n - a);
+}
+// the exponent e of m = f * 2^e with 0.5 <= f < 1, from m's binary32 fields (0 for m = 0; m >= 0,
+// finite; subnormal m from its leading bit)
+__device__ __forceinline__ int vec_exponent(float m) {
+  const uint32_t b = __float_as_uint(m) & 0x7fffffffu;
+  if (b == 0) return 0;
+  const int be = (int)(b >> 23);
+  if (be > 0) return be - 126;
+  return (31 - __clz((int)b)) - 148;
+}
+
+// Splitting group by group: each group is split scaled by its own exponent e_g (quant_vals(v,
+// -e_g)), then, once the vector's exponent e is known (the largest e_g), its s is multiplied by
+// 2^(e_g - e) (rescale_group): the same pieces and s as splitting the group scaled by 2^-e, without
+// keeping the values.  kNoExp stands for the exponent of an all-zero group.
+constexpr int kNoExp = -100000;
+__device__ __forceinline__ int group_exponent(float m) { return m > 0.f ? vec_exponent(m) : kNoExp; }
+__device__ __forceinline__ int vector_exponent(int e_max) { return e_max == kNoExp ? 0 : e_max; }
+template <int QT>
+__device__ __forceinline__ void rescale_group(XQ<QT>& q, int e_g, int e) {
+  q.sf = e_g - e >= -100 ? scale2(q.sf, e_g - e) : 0.f;  // groups below 2^-100 of the vector: zero
+}
+
+// the kW values of one group (kCoherent: read through L2 only, for values other blocks wrote)
 template <int QT, bool kCoherent = false>
-__device__ __forceinline__ XQ<QT> quant_vec(const float* __restrict__ vp) {
-  constexpr int kW = Vec<QT>::kW;
-  float v[kW];
+__device__ __forceinline__ void load_group(const float* __restrict__ vp, float (&v)[Vec<QT>::kW]) {
 #pragma unroll
-  for (int i = 0; i < kW / 4; ++i) {
+  for (int i = 0; i < Vec<QT>::kW / 4; ++i) {
     const float4 f =
         kCoherent ? __ldcg(reinterpret_cast<const float4*>(vp) + i) : __ldg(reinterpret_cast<const float4*>(vp) + i);
     v[4 * i] = f.x;
@@ -128,10 +163,28 @@ __device__ __forceinline__ XQ<QT> quant_vec(const float* __restrict__ vp) {
     v[4 * i + 2] = f.z;
     v[4 * i + 3] = f.w;
   }
+}
+
+template <int QT>
+__device__ __forceinline__ float group_absmax(const float (&v)[Vec<QT>::kW]) {
+  float m = 0.f;
+#pragma unroll
+  for (int j = 0; j < Vec<QT>::kW; ++j) m = fmaxf(m, fabsf(v[j]));
+  return m;
+}
+
+// the pieces of one group, after multiplying its values by 2^ne (ne = -e of the whole vector)
+template <int QT>
+__device__ __forceinline__ XQ<QT> quant_vals(const float (&v0)[Vec<QT>::kW], int ne) {
+  constexpr int kW = Vec<QT>::kW;
+  float v[kW];
+  const float sa = pow2i(ne / 2), sb = pow2i(ne - ne / 2);
+#pragma unroll
+  for (int j = 0; j < kW; ++j) v[j] = v0[j] * sa * sb;
   float m = 0.f;
 #pragma unroll
   for (int j = 0; j < kW; ++j) m = fmaxf(m, fabsf(v[j]));
-  const float inv = m > 0.f ? 127.f / m : 0.f;
+  const float inv = m > 0x1p-100f ? 127.f / m : 0.f;
   XQ<QT> r;
   int s1 = 0, s2 = 0, s3 = 0;
 #pragma unroll
@@ -158,7 +211,7 @@ __device__ __forceinline__ XQ<QT> quant_vec(const float* __restrict__ vp) {
   constexpr int off = QT == kQ8 ? 128 : 8;
   r.k12 = off * (s1 * 127 + s2);
   r.k3 = off * s3;
-  r.sf = m / 127.f / 16129.f;
+  r.sf = inv > 0.f ? m / 127.f / 16129.f : 0.f;
   return r;
 }
 

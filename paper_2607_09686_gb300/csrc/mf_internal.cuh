@@ -13,6 +13,7 @@ namespace mf {
 constexpr int kMaxTopK = 8;
 constexpr int kMaxExperts = 1024;
 constexpr int kTimerClasses = 7;
+constexpr uint64_t kDefaultWaitNs = 1000000000ull;  // bounded device waits give up after 1 s by default
 enum TimerClass { kTRouter = 0, kTResolve = 1, kTMaterialize = 2, kTGateUp = 3, kTDown = 4, kTPrefill = 5, kTFfn = 6 };
 
 // Layout of one expert slot, identical in the pinned pack and in the HBM pool: row records.
@@ -73,8 +74,10 @@ struct Dev {
   uint8_t* xt;         // x tiles:  t * (H / 32) + kk
   uint8_t* ht;         // h tiles:  t * (I / 32) + kk
   uint8_t* stage;      // [S_alloc] payloads: a wave's misses staged while the previous wave computes (T_max > 1)
-  unsigned* work;      // [4]           arrival counter (64-bit) of the fused one-token FFN kernel
+  unsigned long long* work;  // [16]     arrival counter of the fused one-token FFN kernel (word 0)
   unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
+  uint64_t wait_ns;    // time limit of every bounded device wait (mf_wait_limit)
+  int hold;            // test hold (mf_test_hold): the fused FFN's producer issues no copies
 };
 
 // ---- shared-memory pipeline primitives (mbarrier + bulk asynchronous copy, PTX ISA 8.x)
@@ -99,13 +102,61 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait for the phase with the given parity; false after `limit` polls (an error, never a
-// hang: the caller records it and stops using the pipeline).
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint32_t limit = (1u << 26)) {
-  for (uint32_t i = 0; i < limit; ++i)
-    if (mbar_try_wait(bar, parity)) return true;
+// Nanoseconds of the GPU's global timer.
+__device__ __forceinline__ uint64_t gtimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Poll-count backstop of every bounded wait, should the global timer not advance.
+constexpr uint32_t kWaitPolls = 1u << 26;
+// try_wait that may suspend the thread for up to `hint_ns` (it resumes as soon as the phase
+// completes): a waiting warp then takes no issue slots from the warps doing the work.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase with the given parity; false once `limit_ns` nanoseconds have passed
+// since the first failed poll (an error, never a hang: the caller records it and stops using the
+// pipeline).  Between polls the thread sleeps in the barrier (at most 20 us per poll).
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = gtimer_ns();
+  for (uint32_t i = 0; i < kWaitPolls; ++i) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (gtimer_ns() - t0 > limit_ns) return false;
+  }
   return false;
 }
+// Bounded wait until the 64-bit counter reaches `target` (acquire: what the adders released
+// before their additions is visible afterwards); false once `limit_ns` nanoseconds have passed.
+__device__ __forceinline__ bool counter_wait(const unsigned long long* cnt, unsigned long long target,
+                                             uint64_t limit_ns) {
+  uint64_t t0 = 0;
+  for (uint32_t i = 0; i < kWaitPolls; ++i) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(cnt) : "memory");
+    if (v >= target) return true;
+    if (i == 0) t0 = gtimer_ns();
+    if (i >= 32) {
+      if (gtimer_ns() - t0 > limit_ns) return false;
+      __nanosleep(32);
+    }
+  }
+  return false;
+}
+// Programmatic dependent launch (PTX griddepcontrol).  pdl_wait: block until the grid this launch
+// depends on has completed and its memory operations are visible (returns at once when the
+// launch was not programmatic); everything before it may overlap the predecessor's tail and must
+// touch no global memory the predecessor or the caller's earlier work could write.
+// pdl_trigger: allow the dependent launch to be scheduled (its blocks start as SMs free up).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 // bulk copy global -> this CTA's shared memory, completing `bytes` on the mbarrier
 // (addresses 16-byte aligned, bytes a multiple of 16)
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {

@@ -4,7 +4,10 @@
 // but without a context: the weights are the caller's, and the scratch the kernels pass
 // between each other (h, the SwiGLU activations, plus a few small index tables) lives in the
 // file-scope array below instead of in a context's device allocation.
+#include <atomic>
+#include <cstddef>
 #include <cstring>
+#include <mutex>
 
 #include "mf_internal.cuh"
 
@@ -27,12 +30,17 @@ constexpr size_t kNoAllocBytes = kTablesOff + ((sizeof(NoAllocTables) + 255) & ~
 static __device__ __align__(256) unsigned char g_noalloc[kNoAllocBytes];
 
 constexpr int kMaxDevices = 64;
-unsigned char* g_base[kMaxDevices];  // device address of g_noalloc, per device (set up once)
+std::atomic<unsigned char*> g_base[kMaxDevices];  // device address of g_noalloc, per device (set up once)
+std::mutex g_setup_mu;
 
 // Once per device, with that device current: the array's device address (host code only has a
-// stand-in for the symbol) and the constant index tables.
+// stand-in for the symbol) and the constant index tables.  Host threads that make their first
+// call at the same time take turns (the lock); the address is published only after the tables
+// have reached the device, so a first call on any stream reads complete tables.
 int setup(int dev) {
-  if (g_base[dev]) return MF_OK;
+  if (g_base[dev].load(std::memory_order_acquire)) return MF_OK;
+  std::lock_guard<std::mutex> lock(g_setup_mu);
+  if (g_base[dev].load(std::memory_order_relaxed)) return MF_OK;
   void* p = nullptr;
   cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc);
   if (e != cudaSuccess) return MF_E_CUDA;
@@ -49,7 +57,8 @@ int setup(int dev) {
   t.err = 0;
   e = cudaMemcpyToSymbol(g_noalloc, &t, sizeof(t), kTablesOff, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return MF_E_CUDA;
-  g_base[dev] = static_cast<unsigned char*>(p);
+  if ((e = cudaDeviceSynchronize()) != cudaSuccess) return MF_E_CUDA;  // the tables have landed
+  g_base[dev].store(static_cast<unsigned char*>(p), std::memory_order_release);
   return MF_OK;
 }
 
@@ -90,8 +99,9 @@ extern "C" int mf_expert_ffn_noalloc(const mf_model_t* model, const void* expert
   d.S_active = m.top_k;
   d.T_max = 1;
   d.lay = make_layout(m);
+  d.wait_ns = kDefaultWaitNs;
   d.pool = static_cast<uint8_t*>(const_cast<void*>(experts));  // expert j's slot at j * stride
-  unsigned char* base = g_base[dev];
+  unsigned char* base = g_base[dev].load(std::memory_order_acquire);
   NoAllocTables* t = reinterpret_cast<NoAllocTables*>(base + kTablesOff);
   d.h = reinterpret_cast<float*>(base);
   d.uslot = t->ident;
@@ -111,4 +121,20 @@ extern "C" int mf_expert_ffn_noalloc(const mf_model_t* model, const void* expert
     if (launch_down_single(d, 0, y, s) != cudaSuccess) return MF_E_CUDA;
   }
   return MF_OK;
+}
+
+extern "C" int mf_expert_ffn_noalloc_check(void) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return MF_E_CUDA;
+  if (!g_base[dev].load(std::memory_order_acquire)) return MF_OK;  // no call has run on this device
+  if (cudaDeviceSynchronize() != cudaSuccess) return MF_E_CUDA;
+  const size_t off = kTablesOff + offsetof(NoAllocTables, err);
+  unsigned err = 0;
+  if (cudaMemcpyFromSymbol(&err, g_noalloc, sizeof(err), off, cudaMemcpyDeviceToHost) != cudaSuccess) return MF_E_CUDA;
+  if (!err) return MF_OK;
+  const unsigned zero = 0;
+  if (cudaMemcpyToSymbol(g_noalloc, &zero, sizeof(zero), off, cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaDeviceSynchronize() != cudaSuccess)
+    return MF_E_CUDA;
+  return MF_E_TIMEOUT;
 }

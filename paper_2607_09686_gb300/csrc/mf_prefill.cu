@@ -53,7 +53,6 @@ constexpr int kStages = 4;  // operand stages (A + B tiles)
 constexpr int kRaw = 3;     // raw-code ring slots
 constexpr uint32_t kTile = kBM * kBK * 2;  // one bf16 tile: 128 rows x 32 k = 8 KiB
 constexpr uint32_t kBTile = 2 * kTile;     // B hi + lo, one bulk copy
-constexpr uint32_t kWaitLimit = 1u << 26;
 
 // warp roles of the 448-thread CTA
 constexpr int kConvWarps = 8;  // warps 0-7: dequantise A tiles
@@ -288,7 +287,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
   // bounded wait; false (and the block's flag and the device error word set) once any wait gave up
   auto wait = [&](uint64_t* bar, uint32_t parity, unsigned code) -> bool {
     if (*s_flag) return false;
-    if (mbar_wait(bar, parity, kWaitLimit)) return true;
+    if (mbar_wait(bar, parity, d.wait_ns)) return true;
     *s_flag = 1;
     atomicExch(d.err, code);
     return false;
@@ -433,7 +432,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
       }
       // nothing may be in flight when the tensor memory is freed
       mma_commit(drain);
-      if (!mbar_wait(drain, 0, kWaitLimit)) atomicExch(d.err, 10u);
+      if (!mbar_wait(drain, 0, d.wait_ns)) atomicExch(d.err, 10u);
     }
   } else {
     // ================= epilogue: accumulator j & 1 -> outputs

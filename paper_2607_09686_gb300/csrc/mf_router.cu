@@ -131,6 +131,8 @@ __global__ void __launch_bounds__(kThreadsR)
   const int wpe = epc >= kWarpsR ? 1 : kWarpsR / epc;  // warps per expert
   const int ew = kWarpsR / wpe;                         // experts per pass
   const int part = warp % wpe, n4 = H / 4;
+  // a programmatic launch may begin during the previous kernel: nothing above touched global memory
+  pdl_wait();
   float4 pre[kChunk];
   if (e0 + warp / wpe < e1 && warp / wpe < ew) w_preload(wr + (size_t)(e0 + warp / wpe) * H, n4, part * 32 + lane, wpe * 32, pre);
   {  // x may be pinned host memory read over the CPU-GPU link: once per block
@@ -204,6 +206,8 @@ __global__ void __launch_bounds__(kThreadsR)
       }
     }
   }
+  // the logits are stored: the expert FFN (a programmatic launch) may start its prologue
+  pdl_trigger();
   // every block's logits stores, before block 0 reads them; the other blocks leave
   asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
   if (rank != 0) return;
@@ -497,7 +501,7 @@ cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const f
   cfg.blockDim = dim3(kThreadsR);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
@@ -517,6 +521,19 @@ cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const f
   }
   cfg.gridDim = dim3(nc, T);
   attr[0].val.clusterDim.x = nc;
+  // programmatic: the launch may begin while the previous kernel of the stream finishes (the
+  // kernel waits for it before touching global memory); plain where the driver refuses that
+  static bool pdl_ok = true;
+  if (pdl_ok) {
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.numAttrs = 2;
+    e = cudaLaunchKernelEx(&cfg, k_router, d, x, wr, bias, T, layer, T == 1 ? 1 : 0, x_copy, nc);
+    if (e == cudaSuccess) return e;
+    cudaGetLastError();
+    pdl_ok = false;
+    cfg.numAttrs = 1;
+  }
   e = cudaLaunchKernelEx(&cfg, k_router, d, x, wr, bias, T, layer, T == 1 ? 1 : 0, x_copy, nc);
   return e;
 }

@@ -25,8 +25,13 @@ def compare_outputs(got: np.ndarray, ref: np.ndarray) -> dict:
     rms = np.sqrt(np.mean(ref ** 2, axis=1, keepdims=True))
     err = np.abs(got - ref)
     bound = ATOL_RMS * rms + RTOL * np.abs(ref)
-    return dict(ratio=float((err / bound).max()), max_abs=float(err.max()),
-                max_abs_over_rms=float((err / rms).max()),
+    # an all-zero reference row must be matched exactly (its bound is 0); NaN never passes
+    ratio = np.where(err == 0, 0.0, err / np.where(bound > 0, bound, 1e-300))
+    ratio = np.where(np.isfinite(got), ratio, np.inf)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        rel_rms = np.where(rms > 0, err / np.where(rms > 0, rms, 1), np.where(err == 0, 0.0, np.inf))
+    return dict(ratio=float(ratio.max()), max_abs=float(err.max()),
+                max_abs_over_rms=float(rel_rms.max()),
                 literal_fail_frac=float(np.mean(err > 2e-3 + 1e-2 * np.abs(ref))))
 
 
@@ -52,17 +57,21 @@ class Shape:
 
 
 class Payloads:
-    """Canonical payloads regenerated on demand (the oracle's view of the pack)."""
+    """Canonical payloads regenerated on demand (the oracle's view of the pack).  `edit`, if
+    given, is applied to every generated payload (layer, expert, bytes) -> bytes: the same edited
+    bytes go into the context's pack (Ctx(..., edit=...)) and to the oracle."""
 
-    def __init__(self, shape: Shape):
+    def __init__(self, shape: Shape, edit=None):
         self.s = shape
+        self.edit = edit
         self._cache = {}
 
     def get(self, layer: int, expert: int) -> np.ndarray:
         key = (layer, expert)
         if key not in self._cache:
             s = self.s
-            self._cache[key] = synth.payload(s.model_seed, layer, expert, s.hidden, s.inter, s.qtype)
+            p = synth.payload(s.model_seed, layer, expert, s.hidden, s.inter, s.qtype)
+            self._cache[key] = p if self.edit is None else self.edit(layer, expert, p)
         return self._cache[key]
 
     def for_layer(self, layer: int, experts) -> list:
@@ -73,7 +82,7 @@ class Payloads:
 class Ctx:
     """A context of the CUDA library with its pack filled from the seeded generator."""
 
-    def __init__(self, shape: Shape, slots: int, max_tokens: int, device: int = 0, workers: int = 8):
+    def __init__(self, shape: Shape, slots: int, max_tokens: int, device: int = 0, workers: int = 8, edit=None):
         import torch
         import paper_2607_09686_gb300 as mf
         self.mf, self.torch, self.s = mf, torch, shape
@@ -87,6 +96,8 @@ class Ctx:
         def put(le):
             buf = np.empty(n, np.uint8)
             synth.payload(shape.model_seed, le[0], le[1], shape.hidden, shape.inter, shape.qtype, out=buf)
+            if edit is not None:
+                buf = edit(le[0], le[1], buf)
             mf.mf_pack_put(self.h, le[0], le[1], buf)
 
         jobs = [(l, e) for l in range(shape.n_layers) for e in range(shape.n_experts)]

@@ -70,15 +70,52 @@ def test_noalloc_ffn_matches_moe_forward_on_two_calls(shape):
             if t == 1:  # after the first call has set the device up, a call changes no allocation
                 assert torch.cuda.mem_get_info(dev)[0] == free0
             assert_outputs_close(yd.cpu().numpy(), y_ref, f"call {t}")
+        assert mf.mf_expert_ffn_noalloc_check() == mf.MF_OK  # no bounded wait gave up
     finally:
         ctx.close()
+
+
+def _oracle_ffn(payloads, g, x, H, I, q):
+    """y = sum_j g_j FFN_j(x) in fp64 (the oracle's expert FFN), rounded once to fp32."""
+    import oracle
+    acc = np.zeros(H, np.float64)
+    for j, p in enumerate(payloads):
+        yj, _ = oracle.expert_ffn(p, q, H, I, x)
+        acc += np.float64(g[j]) * yj
+    return acc.astype(np.float32)[None]
+
+
+@pytest.mark.parametrize("shape", [(256, 2048, 4, synth.Q8_0),    # the one-warp-per-row kernels
+                                   (256, 4096, 8, synth.Q4_0)],   # top_k * inter = 32768: the limit
+                         ids=["q8_0_unpipelined", "q4_0_at_limit"])
+def test_noalloc_ffn_against_the_oracle(shape):
+    """Shapes the pipelined kernels do not take (h of 2048 / 4096 values per expert) run the other
+    kernel pair; the largest accepted size fills the static scratch exactly."""
+    import torch
+    import paper_2607_09686_gb300 as mf
+    H, I, k, q = shape
+    model = mf.Model(1, H, k, k, I, q)
+    dev = torch.device("cuda:0")
+    pays = [synth.payload(9, 0, e, H, I, q) for e in range(k)]
+    experts = np.concatenate([slot_image(p, H, I, q) for p in pays])
+    ed = torch.from_numpy(experts).to(dev)
+    for t in range(2):  # two calls in a row
+        x = synth.activations(13, 0, 0, t, 1, H)
+        g = np.random.default_rng(t).dirichlet(np.ones(k)).astype(np.float32)
+        yd = torch.full((1, H), float("nan"), device=dev)
+        mf.mf_expert_ffn_noalloc(model, ed, torch.from_numpy(g).to(dev), torch.from_numpy(x).to(dev), yd)
+        torch.cuda.synchronize()
+        assert_outputs_close(yd.cpu().numpy(), _oracle_ffn(pays, g, x[0], H, I, q), f"{shape} call {t}")
+    assert mf.mf_expert_ffn_noalloc_check() == mf.MF_OK
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch():
     import torch
     import paper_2607_09686_gb300 as mf
-    big = mf.Model(1, 2048, 8, 8, 4608, synth.Q8_0)  # 8 * 4608 > 32768 floats of h
     buf = torch.zeros(16, device="cuda")
-    with pytest.raises(mf.MFError) as e:
-        mf.mf_expert_ffn_noalloc(big, buf, buf, buf, buf)
-    assert e.value.status == mf.MF_E_INVAL
+    # Q4_0, top_k 8, inter 4128: a valid expert shape whose h (33024 floats) exceeds the scratch
+    # (Q8_0 shapes past the limit are already rejected as shapes)
+    for big in (mf.Model(1, 256, 8, 8, 4128, synth.Q4_0), mf.Model(1, 2048, 8, 8, 4608, synth.Q8_0)):
+        with pytest.raises(mf.MFError) as e:
+            mf.mf_expert_ffn_noalloc(big, buf, buf, buf, buf)
+        assert e.value.status == mf.MF_E_INVAL
