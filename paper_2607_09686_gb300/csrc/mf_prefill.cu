@@ -286,6 +286,7 @@ __global__ void __launch_bounds__(kThreadsW, 1)
 
   // bounded wait; false (and the block's flag and the device error word set) once any wait gave up
   auto wait = [&](uint64_t* bar, uint32_t parity, unsigned code) -> bool {
+    if (mbar_try_wait(bar, parity)) return true;  // the common case: no flag read on the fast path
     if (*s_flag) return false;
     if (mbar_wait(bar, parity, d.wait_ns)) return true;
     *s_flag = 1;
@@ -350,7 +351,9 @@ __global__ void __launch_bounds__(kThreadsW, 1)
       if (++stage == kStages) stage = 0, sph ^= 1;
     }
   } else if (warp == kProdWarp) {
-    // ================= producer: TMA boxes of codes and scales, bulk B tile
+    // ================= producer (lane 0; the warp's other lanes have no role): TMA boxes of codes
+    // and scales, bulk B tile
+    if (lane == 0) {
     const uint8_t* tiles = NT == 2 ? d.xt : d.ht;
     int y0 = 0, z0 = 0;    // the unit's TMA coordinates: first row, slot plane
     size_t b0 = 0;         // its first B tile
@@ -366,12 +369,12 @@ __global__ void __launch_bounds__(kThreadsW, 1)
         const int a0 = d.asg_off[un.u] + un.tb * kBN;
         b_bytes = (uint32_t)n_eff(min(kBN, d.asg_off[un.u + 1] - a0)) * (kBK * 2);
       }
-      if (s >= kRaw && !warp_wait(&raw_free[slot], rph ^ 1, 3u)) break;
-      if (s >= kStages && !warp_wait(&mma_done[stage], sph ^ 1, 4u)) break;
+      if (s >= kRaw && !wait(&raw_free[slot], rph ^ 1, 3u)) break;
+      if (s >= kStages && !wait(&mma_done[stage], sph ^ 1, 4u)) break;
       unsigned char* raw = smem + PL::kOffRaw + slot * PL::kRawSlot;
       const bool group = (kk & (kGroup - 1)) == 0;
       if (group) gb ^= 1;
-      if (lane == 0) {
+      {
         mbar_arrive_tx(&full[slot], NT * kBM * CB + 2 * b_bytes + (group ? PL::kScaleBuf : 0u));
 #pragma unroll
         for (int tn = 0; tn < NT; ++tn)
@@ -390,10 +393,10 @@ __global__ void __launch_bounds__(kThreadsW, 1)
         bulk_g2s(bdst, bsrc, b_bytes, &full[slot]);                  // hi: the first n_eff columns
         bulk_g2s(bdst + kTile, bsrc + kTile, b_bytes, &full[slot]);  // lo
       }
-      __syncwarp();
       if (++kk == nk) kk = 0, ++j;
       if (++slot == kRaw) slot = 0, rph ^= 1;
       if (++stage == kStages) stage = 0, sph ^= 1;
+    }
     }
   } else if (warp == kMmaWarp) {
     // ================= MMA issue (one thread)
