@@ -432,6 +432,9 @@ def extras(args, line, torch, mf, synth, device, cfg, ctx, dec, flush, stream, t
                          "link_ms_per_step_at_h2d": round(link_ms, 3),
                          "link_share_of_step": round(link_ms / line["ms_per_step"], 4),
                          "h2d_how": "pinned host -> device cudaMemcpyAsync of 1 GiB, best of 10, this run"})
+    _guard(line["copy"], "placement", host_placement)
+    if not args.no_link:
+        _guard(line["copy"], "in_kernel_link", lambda: link_measurement(torch, mf, synth, cfg, ctx, dec, stream, h2d))
     if not args.no_resident:
         _guard(line["roofline"], "resident", lambda: resident_measurement(torch, mf, ctx, dec, flush, stream, args.steps,
                                                                           rf_bytes, hbm))
@@ -453,6 +456,59 @@ def extras_other_contexts(args, line, torch, mf, synth, device):
         _guard(line, "batch64", lambda: batch64_measurement(torch, mf, synth, device))
     if not args.no_l4e64:
         _guard(line, "l4e64", lambda: l4e64_measurement(torch, mf, synth, device, args.steps))
+
+
+def host_placement() -> dict:
+    """Where the pinned pack sits relative to the GPU: the host's NUMA nodes (sysfs) and the GPU's
+    (the PCI device's numa_node).  The pack is allocated by the calling thread (cudaHostAlloc), so
+    its pages land on that thread's node."""
+    nodes = sorted(int(n[4:]) for n in os.listdir("/sys/devices/system/node") if n[4:].isdigit())
+    cpus = {n: open(f"/sys/devices/system/node/node{n}/cpulist").read().strip() for n in nodes}
+    try:
+        bus = subprocess.run(["nvidia-smi", "--id=0", "--query-gpu=pci.bus_id", "--format=csv,noheader"],
+                             capture_output=True, text=True).stdout.strip().lower()
+    except Exception:
+        bus = ""
+    dev = bus[4:] if len(bus) > 12 else bus  # 00000000:00:07.0 -> 0000:00:07.0
+    try:
+        gnode = int(open(f"/sys/bus/pci/devices/{dev}/numa_node").read())
+    except Exception:
+        gnode = None
+    return {"numa_nodes": nodes, "cpus_per_node": cpus, "gpu_pci": dev, "gpu_numa_node": gnode,
+            "pack": "cudaHostAlloc(mapped | portable) by the calling thread: pages on its node"
+                    + (" (the only node)" if len(nodes) == 1 else "")}
+
+
+def link_measurement(torch, mf, synth, cfg, ctx, dec, stream, h2d_gbs: float, reps: int = 3) -> dict:
+    """The fused FFN launch when every one of its k experts misses: layer 0 with all 128 slots in
+    use from a cold cache, 16 calls whose planted routes are disjoint sets of 8 experts, so each
+    launch pulls 8 payloads (40.1 MB) over the CPU-GPU link inside the kernel.  CUDA events around
+    each FFN launch; bytes = misses x payload (the ncu sysmem sector count of such a launch agrees
+    to 0.1 %)."""
+    E, k, H = cfg.n_experts, cfg.top_k, cfg.hidden
+    n = E // k
+    routes = np.arange(n * k, dtype=np.int32).reshape(n, k)
+    x = dec.x[:n, 0].contiguous()
+    b = torch.from_numpy(synth.plant_bias(routes, E)).to(x.device)
+    y = torch.empty(n, H, device=x.device)
+    rates = []
+    for _ in range(reps):
+        mf.mf_reset(ctx, E, stream)
+        mf.mf_timing(ctx, ["ffn_fused"])
+        with torch.cuda.stream(stream):
+            for t in range(n):
+                mf.mf_moe_forward(ctx, 0, x[t], dec.wr[0], b[t], 1, y[t], None, None, stream)
+        tm = mf.mf_timing_read(ctx)["ffn_fused"]
+        st = mf.mf_stats(ctx, 0)
+        rates.append(st["bytes_materialized"] / (tm[0] * 1e-3) / 1e9)
+        assert st["misses"] == n * k
+    mf.mf_timing(ctx, [])
+    assert mf.mf_check(ctx) == 0
+    gbs = max(rates)
+    return {"gbs": round(gbs, 1), "frac_of_h2d": round(gbs / h2d_gbs, 4), "misses_per_launch": k,
+            "bytes_per_launch": int(mf.mf_payload_bytes(mf.Model(1, H, E, k, cfg.inter, cfg.qtype))) * k,
+            "how": f"{n} one-token calls of layer 0 from a cold cache with disjoint planted routes (every "
+                   f"expert misses), CUDA events around each fused FFN launch, best of {reps}"}
 
 
 def resident_measurement(torch, mf, ctx, dec, flush, stream, steps, bytes_per_launch, hbm):
@@ -1054,6 +1110,7 @@ def main():
     ap.add_argument("--no-tuner", action="store_true", help="skip the cache-size tuner against measured steps")
     ap.add_argument("--no-spec", action="store_true", help="skip the speculative verification-width accounting")
     ap.add_argument("--no-l4e64", action="store_true", help="skip the 4-layer workload")
+    ap.add_argument("--no-link", action="store_true", help="skip the all-miss in-kernel link measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle

@@ -136,21 +136,30 @@ int mf_tune_cache(const mf_model_t* model, const mf_plan_req_t* req, const int32
  * needed.  Fills *out even when rejecting; returns MF_E_BUDGET if L > budget. */
 int mf_plan(const mf_model_t* model, const mf_plan_req_t* req, mf_plan_t* out);
 
-/* Create a context on CUDA device `device`: allocates the pinned host pack
- * (n_layers * n_experts payloads), the HBM slot pool (n_layers * S payloads), the slot
- * table and the scratch for plan->max_tokens.  Refuses a rejected plan (MF_E_BUDGET).
- * The pack is empty: fill it with mf_pack_put before the first mf_moe_forward. */
+/* Create a context on CUDA device `device` (section "Split-Pack Representation": routed expert
+ * tensors are held outside fast memory as per-layer, per-expert payloads, and the runtime
+ * materialises only the experts a step needs; section "Native Serving Path": bounded per-layer
+ * slots).  Allocates the pinned host pack (n_layers * n_experts payloads: the split-pack), the
+ * HBM slot pool (n_layers * S payloads), the slot table and the scratch for plan->max_tokens.
+ * Refuses a rejected plan (MF_E_BUDGET); MF_E_INVAL for an invalid model or a plan that does not
+ * belong to it; MF_E_OOM when an allocation fails (nothing is left allocated).  The pack is
+ * empty: fill it with mf_pack_put before the first mf_moe_forward (MF_E_STATE until then). */
 int mf_create(mf_ctx_t** out, const mf_model_t* model, const mf_plan_t* plan, int device);
 
-/* Copy one expert's canonical GGUF payload (host memory, `bytes` must equal
- * payload_bytes) into the pinned pack, repacked so quantised codes and scales are
- * 16-byte aligned (the same bytes, regrouped; accounting stays at payload_bytes).
- * The caller may free `payload` when the call returns.  Host only, synchronous; calls for
- * distinct (layer, expert) pairs may run concurrently from several host threads. */
+/* Copy one expert's canonical GGUF payload (host memory, `bytes` must equal payload_bytes)
+ * into its place in the pinned split-pack (section "Split-Pack Representation": one payload per
+ * (layer, expert), gate, up and down tensors together), repacked into row records so that
+ * quantised codes and scales are 16-byte aligned and the rows a kernel computes together are
+ * contiguous (the same bytes, regrouped; accounting stays at payload_bytes).  The caller may free
+ * `payload` when the call returns.  MF_E_INVAL for a NULL payload, a layer or expert out of range
+ * or a wrong size.  Host only, synchronous; calls for distinct (layer, expert) pairs may run
+ * concurrently from several host threads. */
 int mf_pack_put(mf_ctx_t* ctx, int layer, int expert, const void* payload, uint64_t bytes);
 
 /* mf_create followed by mf_pack_put of payloads[layer * n_experts + expert] (host
- * pointers, each payload_bytes long) for every layer and expert. */
+ * pointers, each payload_bytes long) for every layer and expert: the whole split-pack loaded
+ * (section "Split-Pack Representation").  MF_E_INVAL if any pointer is NULL; on any failure
+ * nothing is left allocated and *out is NULL. */
 int mf_load_pack(mf_ctx_t** out, const mf_model_t* model, const mf_plan_t* plan,
                  const void* const* payloads, int device);
 
