@@ -456,6 +456,8 @@ def extras_other_contexts(args, line, torch, mf, synth, device):
         _guard(line, "batch64", lambda: batch64_measurement(torch, mf, synth, device))
     if not args.no_l4e64:
         _guard(line, "l4e64", lambda: l4e64_measurement(torch, mf, synth, device, args.steps))
+    if not args.no_disk:
+        _guard(line, "disk", lambda: disk_measurement(torch, mf, synth, device))
 
 
 def host_placement() -> dict:
@@ -934,6 +936,81 @@ def batch64_measurement(torch, mf, synth, device, steps: int = 8, warm: int = 2,
     return out
 
 
+def disk_measurement(torch, mf, synth, device, cache_pct: float = 15.0, reps: int = 2) -> dict:
+    """The disk tier against the pinned pack on the headline workload at 15 % cache (19 slots):
+    the split-pack written to a file (mf_pack_save), a context serving its misses from the file
+    (mf_create_from_file: after the router decides a call's misses, a host function reads them
+    into pinned staging), and the same 96-token decode through both (one graph each, from a cold
+    cache).  Every layer of the model when the file system holds the 31 GB file twice over, else
+    the first layers that fit."""
+    import shutil
+    import tempfile
+    cfg = synth.CONFIGS[WORKLOAD]
+    H, E, k, I, q = cfg.hidden, cfg.n_experts, cfg.top_k, cfg.inter, cfg.qtype
+    pdir = os.environ.get("MF_PACK_DIR", tempfile.gettempdir())
+    per_layer = E * (synth.payload_bytes(H, I, q) + 4096)
+    free = shutil.disk_usage(pdir).free
+    L = min(cfg.n_layers, int(free // 2 // per_layer))
+    if L < 1:
+        return {"skipped": f"{free / 1e9:.1f} GB free in {pdir}"}
+    model = mf.Model(L, H, E, k, I, q)
+    plan = mf.mf_plan(model, mf.PlanReq(cache_pct, 1 << 62, 0, 0, 1, 0))
+    head = _klass(cfg, HEAD_CLASS)
+    path = os.path.join(pdir, f"mawforge_l{L}e{E}.mfpack")
+    stream = torch.cuda.Stream(device)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=device)
+    sub = cfg.__class__(**{**cfg.__dict__, "n_layers": L})
+    xn, bn = decode_inputs(synth, sub, HEAD_SEED, head)
+    x = torch.from_numpy(xn).to(device)
+    b = torch.from_numpy(bn).to(device)
+    wr = torch.from_numpy(np.stack([synth.router_weights(cfg.model_seed, l, E, H) for l in range(L)])).to(device)
+    out = {"workload": f"{WORKLOAD} layers 0-{L - 1} of {cfg.n_layers}, {HEAD_CLASS}, cache {cache_pct:g}% "
+                       f"({plan.slots_per_layer} slots), 96 decode tokens batch 1 from a cold cache",
+           "file_dir": pdir}
+    ctx = mf.mf_create(model, plan, device.index or 0)
+    fh = None
+    try:
+        fill_pack(mf, synth, ctx, sub)
+        t0 = time.perf_counter()
+        mf.mf_pack_save(ctx, path)
+        out["save_s"] = round(time.perf_counter() - t0, 2)
+        out["file_gb"] = round(os.path.getsize(path) / 1e9, 2)
+        fh = mf.mf_create_from_file(model, plan, path, device.index or 0)
+        out["direct_io"] = mf.mf_pack_file_direct(fh)
+        res = {}
+        for name, h in (("pinned_pack", ctx), ("file", fh)):
+            dec = Decoder(torch, mf, h, x, b, wr, stream)
+            g = dec.capture(plan.slots_per_layer)
+            f0 = mf.mf_pack_file_stats(fh) if h == fh else None
+            ms = statistics.mean(replay(torch, stream, g, flush, reps, warm=1))
+            del g
+            st = mf.mf_stats(h, -1)
+            assert mf.mf_check(h) == 0
+            r = {"tokens_per_s": round(N_TOKENS / (ms * 1e-3), 2), "ms_per_step": round(ms, 2),
+                 "misses_per_step": st["misses"], "materialized_gb_per_step": round(st["bytes_materialized"] / 1e9, 3)}
+            if f0 is not None:
+                f1 = mf.mf_pack_file_stats(fh)
+                n = reps + 1
+                r["file_reads_per_step"] = (f1["reads"] - f0["reads"]) // n
+                r["read_s_per_step"] = round((f1["seconds"] - f0["seconds"]) / n, 3)
+                r["read_gbs"] = round((f1["bytes"] - f0["bytes"]) / max(1e-9, f1["seconds"] - f0["seconds"]) / 1e9, 2)
+            res[name] = r
+        out.update(res)
+        out["file_minus_pinned_ms_per_step"] = round(res["file"]["ms_per_step"] - res["pinned_pack"]["ms_per_step"], 2)
+        out["how"] = ("the same graph of the 96-token decode through a context with the pinned pack and through one "
+                      "reading its misses from the split-pack file; mean of the replays after one, each from a cold "
+                      "cache; read seconds on the host clock")
+    finally:
+        if fh:
+            mf.mf_destroy(fh)
+        mf.mf_destroy(ctx)
+        try:
+            os.remove(path)
+        except OSError:
+            pass
+    return out
+
+
 def l4e64_measurement(torch, mf, synth, device, steps: int, cache_pct: float = 35.0) -> dict:
     """The 4-layer workload (hidden 2048, 64 experts, top-8, inter 768, Q8_0; 256 decode tokens
     at batch 1, Zipf 1.1 + 0.6 reuse) at 35 % cache: one graph of its 1024 calls per step from a
@@ -1111,6 +1188,7 @@ def main():
     ap.add_argument("--no-spec", action="store_true", help="skip the speculative verification-width accounting")
     ap.add_argument("--no-l4e64", action="store_true", help="skip the 4-layer workload")
     ap.add_argument("--no-link", action="store_true", help="skip the all-miss in-kernel link measurement")
+    ap.add_argument("--no-disk", action="store_true", help="skip the split-pack file (disk tier) measurement")
     args = ap.parse_args()
     if args.impl == "reference":
         import oracle

@@ -47,6 +47,7 @@ extern "C" {
 #define MF_E_CUDA (-4)   /* a CUDA runtime call or kernel launch failed */
 #define MF_E_STATE (-5)  /* the call is not valid in the context's current state */
 #define MF_E_TIMEOUT (-6) /* a bounded wait inside a kernel gave up (reported by mf_check) */
+#define MF_E_IO (-7)      /* reading a split-pack file failed (reported by mf_check) */
 
 /* ---- quantisation types (GGUF type ids) ---- */
 #define MF_Q4_0 2
@@ -155,6 +156,40 @@ int mf_create(mf_ctx_t** out, const mf_model_t* model, const mf_plan_t* plan, in
  * or a wrong size.  Host only, synchronous; calls for distinct (layer, expert) pairs may run
  * concurrently from several host threads. */
 int mf_pack_put(mf_ctx_t* ctx, int layer, int expert, const void* payload, uint64_t bytes);
+
+/* Write the context's split-pack to a file (section "Split-Pack Representation": the expert
+ * payloads in one pack file with an index of layer, expert, offset, byte count and digest, so the
+ * runtime can address one expert block without reading unrelated weights).  Layout: a 4096-byte
+ * header (magic "MFSPLIT1", version 1, the model, payload bytes, slot-layout bytes, record bytes,
+ * index and record offsets), the index (one 32-byte entry per (layer, expert), layer-major: layer,
+ * expert, record offset, payload bytes, 64-bit FNV-1a digest of the record's bytes), then one
+ * record per payload in the pack's slot layout, each padded to a multiple of 4096 bytes.  Every
+ * payload must have been put (MF_E_STATE otherwise, and for a file-backed context); MF_E_INVAL
+ * for a NULL path or when the file cannot be written (a partial file is removed).  Host only. */
+int mf_pack_save(mf_ctx_t* ctx, const char* path);
+
+/* As mf_create, but the split-pack is the file `path` written by mf_pack_save (the disk tier:
+ * the model stays a disk object; section "Split-Pack Representation", and the Introduction's
+ * memory hierarchy of disk, memory and slots).  No pinned pack is allocated: misses are still
+ * decided on the GPU, and after the kernels that decide them a host function on the call's stream
+ * reads the missed records from the file (all of the call's misses, or a wave's, in parallel
+ * 1 MiB reads, unbuffered where the file system allows it) into pinned staging of max(top_k, S)
+ * records, from which the kernels copy them into their slots over the CPU-GPU link.  Calls are
+ * stream-ordered as usual and may be captured into CUDA graphs (the reads become host nodes).
+ * MF_E_INVAL if the file is missing, truncated, or its header or index do not match the model;
+ * MF_E_OOM if the staging cannot be allocated.  mf_pack_put on such a context returns
+ * MF_E_STATE.  A failed read is reported by mf_check as MF_E_IO. */
+int mf_create_from_file(mf_ctx_t** out, const mf_model_t* model, const mf_plan_t* plan, const char* path,
+                        int device);
+
+/* Reads of a file-backed context since its creation: payload records read, bytes read and the
+ * seconds the reads took (summed over calls, host clock).  MF_E_INVAL for a context without a
+ * file.  Host only; counts only calls the stream has reached. */
+int mf_pack_file_stats(mf_ctx_t* ctx, uint64_t* reads, uint64_t* bytes, double* seconds);
+
+/* 1 if the file-backed context reads its file unbuffered (O_DIRECT), 0 if through the page cache,
+ * MF_E_INVAL for a context without a file. */
+int mf_pack_file_direct(mf_ctx_t* ctx);
 
 /* mf_create followed by mf_pack_put of payloads[layer * n_experts + expert] (host
  * pointers, each payload_bytes long) for every layer and expert: the whole split-pack loaded

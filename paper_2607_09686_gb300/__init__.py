@@ -18,13 +18,14 @@ __all__ = [
     "MFError", "Model", "PlanReq", "Plan", "Stats", "TunePoint", "Q8_0", "Q4_0", "LIB_PATH", "KERNEL_CLASSES",
     "mf_payload_bytes", "mf_plan", "mf_tune_cache", "mf_create", "mf_pack_put", "mf_load_pack", "mf_moe_forward",
     "mf_moe_forward_host", "mf_prefill_threshold", "mf_access_order", "mf_stats", "mf_reset", "mf_trace", "mf_timing", "mf_timing_read", "mf_check", "mf_wait_limit", "mf_test_hold", "mf_expert_ffn_noalloc",
-    "mf_expert_ffn_noalloc_check", "mf_destroy",
+    "mf_expert_ffn_noalloc_check", "mf_pack_save", "mf_create_from_file", "mf_pack_file_stats",
+    "mf_pack_file_direct", "mf_destroy",
     "mf_strerror", "mf_last_cuda_error",
 ]
 
 Q4_0 = 2
 Q8_0 = 8
-MF_OK, MF_E_INVAL, MF_E_BUDGET, MF_E_OOM, MF_E_CUDA, MF_E_STATE, MF_E_TIMEOUT = 0, -1, -2, -3, -4, -5, -6
+MF_OK, MF_E_INVAL, MF_E_BUDGET, MF_E_OOM, MF_E_CUDA, MF_E_STATE, MF_E_TIMEOUT, MF_E_IO = 0, -1, -2, -3, -4, -5, -6, -7
 KERNEL_CLASSES = ("router", "resolve", "materialize", "gateup_swiglu", "down_combine", "prefill_gemm", "ffn_fused")
 
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmawforge.so")
@@ -95,6 +96,11 @@ _sig = {
     "mf_test_hold": (_i32, [_vp, _i32]),
     "mf_expert_ffn_noalloc": (_i32, [ctypes.POINTER(Model), _vp, _vp, _vp, _vp, _vp]),
     "mf_expert_ffn_noalloc_check": (_i32, []),
+    "mf_pack_save": (_i32, [_vp, ctypes.c_char_p]),
+    "mf_create_from_file": (_i32, [ctypes.POINTER(_vp), ctypes.POINTER(Model), ctypes.POINTER(Plan), ctypes.c_char_p,
+                                   _i32]),
+    "mf_pack_file_stats": (_i32, [_vp, ctypes.POINTER(_u64), ctypes.POINTER(_u64), ctypes.POINTER(ctypes.c_double)]),
+    "mf_pack_file_direct": (_i32, [_vp]),
     "mf_destroy": (None, [_vp]),
     "mf_strerror": (ctypes.c_char_p, [_i32]),
     "mf_last_cuda_error": (ctypes.c_char_p, []),
@@ -193,6 +199,34 @@ def mf_pack_put(ctx: int, layer: int, expert: int, payload) -> None:
     _check(_lib.mf_pack_put(ctx, layer, expert, _addr(payload), n), "mf_pack_put")
 
 
+def mf_pack_save(ctx: int, path: str) -> None:
+    """Write the context's split-pack to a file (header, index, one record per payload)."""
+    _check(_lib.mf_pack_save(ctx, os.fsencode(path)), "mf_pack_save")
+
+
+def mf_create_from_file(model: Model, plan: Plan, path: str, device: int = 0) -> int:
+    """A context whose split-pack is the file written by mf_pack_save (misses read from it)."""
+    h = _vp()
+    _check(_lib.mf_create_from_file(ctypes.byref(h), ctypes.byref(model), ctypes.byref(plan), os.fsencode(path),
+                                    device), "mf_create_from_file")
+    return h.value
+
+
+def mf_pack_file_stats(ctx: int) -> dict:
+    """{reads, bytes, seconds} of a file-backed context's reads so far."""
+    r, b, t = _u64(), _u64(), ctypes.c_double()
+    _check(_lib.mf_pack_file_stats(ctx, ctypes.byref(r), ctypes.byref(b), ctypes.byref(t)), "mf_pack_file_stats")
+    return {"reads": int(r.value), "bytes": int(b.value), "seconds": float(t.value)}
+
+
+def mf_pack_file_direct(ctx: int) -> bool:
+    """True if the file-backed context reads its file unbuffered (O_DIRECT)."""
+    rc = _lib.mf_pack_file_direct(ctx)
+    if rc < 0:
+        _check(rc, "mf_pack_file_direct")
+    return rc == 1
+
+
 def mf_load_pack(model: Model, plan: Plan, payloads, device: int = 0) -> int:
     """payloads: sequence of L*E host buffers (numpy uint8), layer-major."""
     arr = (_vp * len(payloads))(*[_addr(p) for p in payloads])
@@ -270,9 +304,10 @@ def mf_timing_read(ctx: int) -> dict:
 
 
 def mf_check(ctx: int) -> int:
-    """0, or MF_E_TIMEOUT if a kernel of this context gave up a bounded wait (returned, not raised)."""
+    """0, MF_E_TIMEOUT if a kernel of this context gave up a bounded wait, or MF_E_IO if a read of
+    its split-pack file failed (returned, not raised)."""
     rc = _lib.mf_check(ctx)
-    if rc not in (MF_OK, MF_E_TIMEOUT):
+    if rc not in (MF_OK, MF_E_TIMEOUT, MF_E_IO):
         _check(rc, "mf_check")
     return rc
 

@@ -203,6 +203,7 @@ void free_ctx(mf_ctx* c) {
   if (c->d.pool) cudaFree(c->d.pool);
   if (c->gemm_scratch) cudaFree(c->gemm_scratch);
   if (c->pack_host) cudaFreeHost(c->pack_host);
+  close_pack_file(c);
   free(c->put_map);
   delete c;
 }
@@ -258,49 +259,10 @@ Layout make_layout(const mf_model_t& m) {
 
 }  // namespace mf
 
-using namespace mf;
-
-extern "C" {
-
-const char* mf_strerror(int status) {
-  switch (status) {
-    case MF_OK: return "ok";
-    case MF_E_INVAL: return "invalid argument";
-    case MF_E_BUDGET: return "static plan rejected: lower bound exceeds the budget";
-    case MF_E_OOM: return "out of memory";
-    case MF_E_CUDA: return "CUDA error";
-    case MF_E_STATE: return "invalid state";
-    case MF_E_TIMEOUT: return "a bounded device-side wait gave up";
-    default: return "unknown status";
-  }
-}
-
-const char* mf_last_cuda_error(void) { return g_cuda_err; }
-
-int mf_payload_bytes(const mf_model_t* model, uint64_t* out) {
-  if (!valid_model(model) || !out) return MF_E_INVAL;
-  *out = canonical_payload_bytes(*model);
-  return MF_OK;
-}
-
-int mf_plan(const mf_model_t* m, const mf_plan_req_t* r, mf_plan_t* out) {
-  if (!valid_model(m) || !r || !out) return MF_E_INVAL;
-  if (!(r->cache_pct >= 0.0 && r->cache_pct <= 100.0) || r->max_tokens < 0 || r->max_tokens > 65535) return MF_E_INVAL;
-  mf_plan_t p;
-  memset(&p, 0, sizeof(p));
-  p.slots_per_layer = slots_for(*m, r->cache_pct);
-  p.payload_bytes = canonical_payload_bytes(*m);
-  p.pool_bytes = (uint64_t)m->n_layers * (uint64_t)p.slots_per_layer * p.payload_bytes;
-  p.lower_bound_bytes = r->common_bytes + p.pool_bytes + r->kv_bytes;
-  p.max_tokens = r->max_tokens > 0 ? r->max_tokens : 1;
-  p.overhead_bytes = overhead_bytes(*m, p.slots_per_layer, p.max_tokens);
-  p.footprint_bytes = p.lower_bound_bytes + p.overhead_bytes;
-  p.accepted = p.lower_bound_bytes <= r->budget_bytes;
-  *out = p;
-  return p.accepted ? MF_OK : MF_E_BUDGET;
-}
-
-int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int device) {
+namespace mf {
+namespace {
+// A context with its pinned pack (with_pack) or, for a file-backed split-pack, without one.
+int create_ctx(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int device, bool with_pack) {
   if (!out || !valid_model(m) || !p) return MF_E_INVAL;
   *out = nullptr;
   if (!p->accepted) return MF_E_BUDGET;
@@ -333,23 +295,25 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
 
   int rc = MF_OK;
   cudaError_t e;
-  const uint64_t pack_bytes = (uint64_t)d.L * d.E * d.lay.stride;
-  e = cudaHostAlloc((void**)&c->pack_host, pack_bytes, cudaHostAllocMapped | cudaHostAllocPortable);
-  if (e != cudaSuccess) {
-    rc = cuda_fail(e, "cudaHostAlloc(pack)");
-    if (rc == MF_E_CUDA) rc = MF_E_OOM;
-    c->pack_host = nullptr;
-    free_ctx(c);
-    return rc;
+  if (with_pack) {
+    const uint64_t pack_bytes = (uint64_t)d.L * d.E * d.lay.stride;
+    e = cudaHostAlloc((void**)&c->pack_host, pack_bytes, cudaHostAllocMapped | cudaHostAllocPortable);
+    if (e != cudaSuccess) {
+      rc = cuda_fail(e, "cudaHostAlloc(pack)");
+      if (rc == MF_E_CUDA) rc = MF_E_OOM;
+      c->pack_host = nullptr;
+      free_ctx(c);
+      return rc;
+    }
+    void* dev_pack = nullptr;
+    e = cudaHostGetDevicePointer(&dev_pack, c->pack_host, 0);
+    if (e != cudaSuccess) {
+      rc = cuda_fail(e, "cudaHostGetDevicePointer");
+      free_ctx(c);
+      return rc;
+    }
+    d.pack = static_cast<const uint8_t*>(dev_pack);
   }
-  void* dev_pack = nullptr;
-  e = cudaHostGetDevicePointer(&dev_pack, c->pack_host, 0);
-  if (e != cudaSuccess) {
-    rc = cuda_fail(e, "cudaHostGetDevicePointer");
-    free_ctx(c);
-    return rc;
-  }
-  d.pack = static_cast<const uint8_t*>(dev_pack);
   c->put_map = static_cast<unsigned char*>(calloc((size_t)d.L * d.E, 1));
   if (!c->put_map) {
     free_ctx(c);
@@ -448,9 +412,76 @@ int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devic
   *out = c;
   return MF_OK;
 }
+}  // namespace
+}  // namespace mf
+
+using namespace mf;
+
+extern "C" {
+
+const char* mf_strerror(int status) {
+  switch (status) {
+    case MF_OK: return "ok";
+    case MF_E_INVAL: return "invalid argument";
+    case MF_E_BUDGET: return "static plan rejected: lower bound exceeds the budget";
+    case MF_E_OOM: return "out of memory";
+    case MF_E_CUDA: return "CUDA error";
+    case MF_E_STATE: return "invalid state";
+    case MF_E_TIMEOUT: return "a bounded device-side wait gave up";
+    case MF_E_IO: return "reading the split-pack file failed";
+    default: return "unknown status";
+  }
+}
+
+const char* mf_last_cuda_error(void) { return g_cuda_err; }
+
+int mf_payload_bytes(const mf_model_t* model, uint64_t* out) {
+  if (!valid_model(model) || !out) return MF_E_INVAL;
+  *out = canonical_payload_bytes(*model);
+  return MF_OK;
+}
+
+int mf_plan(const mf_model_t* m, const mf_plan_req_t* r, mf_plan_t* out) {
+  if (!valid_model(m) || !r || !out) return MF_E_INVAL;
+  if (!(r->cache_pct >= 0.0 && r->cache_pct <= 100.0) || r->max_tokens < 0 || r->max_tokens > 65535) return MF_E_INVAL;
+  mf_plan_t p;
+  memset(&p, 0, sizeof(p));
+  p.slots_per_layer = slots_for(*m, r->cache_pct);
+  p.payload_bytes = canonical_payload_bytes(*m);
+  p.pool_bytes = (uint64_t)m->n_layers * (uint64_t)p.slots_per_layer * p.payload_bytes;
+  p.lower_bound_bytes = r->common_bytes + p.pool_bytes + r->kv_bytes;
+  p.max_tokens = r->max_tokens > 0 ? r->max_tokens : 1;
+  p.overhead_bytes = overhead_bytes(*m, p.slots_per_layer, p.max_tokens);
+  p.footprint_bytes = p.lower_bound_bytes + p.overhead_bytes;
+  p.accepted = p.lower_bound_bytes <= r->budget_bytes;
+  *out = p;
+  return p.accepted ? MF_OK : MF_E_BUDGET;
+}
+
+int mf_create(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int device) {
+  return create_ctx(out, m, p, device, true);
+}
+
+int mf_create_from_file(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, const char* path, int device) {
+  if (!out || !path) return MF_E_INVAL;
+  *out = nullptr;
+  mf_ctx_t* c = nullptr;
+  int rc = create_ctx(&c, m, p, device, false);
+  if (rc) return rc;
+  DevGuard guard(device);
+  if ((rc = open_pack_file(c, path)) != MF_OK) {
+    free_ctx(c);
+    return rc;
+  }
+  c->n_put = (int64_t)c->d.L * c->d.E;  // every payload is in the file
+  *out = c;
+  return MF_OK;
+}
+
 
 int mf_pack_put(mf_ctx_t* c, int layer, int expert, const void* payload, uint64_t bytes) {
   if (!c || !payload || layer < 0 || layer >= c->d.L || expert < 0 || expert >= c->d.E) return MF_E_INVAL;
+  if (!c->pack_host) return MF_E_STATE;  // a file-backed split-pack is read-only
   const Layout& l = c->d.lay;
   if (bytes != l.canonical) return MF_E_INVAL;
   const mf_model_t& m = c->model;
@@ -510,6 +541,7 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   const bool gemm = T > 1 && c->prefill_min_t > 0 && T >= c->prefill_min_t;
 
   if (T == 1 && c->ffn_fused) {  // one launch: expert FFN, with the misses materialised inside
+    if (c->file) MF_CUDA(enqueue_file_reads(c, layer, 0, true, s));  // the misses, file -> staging
     timer_mark(c, kTFfn, 0, s);
     MF_CUDA(launch_ffn_single(d, layer, x, y, s));
     timer_mark(c, kTFfn, 1, s);
@@ -524,13 +556,14 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   // Materialisation on the side stream.  One wave: its misses straight into their slots, then
   // the compute.  Several waves: wave 0 as above; wave w + 1's misses are staged while wave w
   // computes (their slots may still be read by it) and committed to the slots once it is done.
-  const bool staged = n_waves > 1 && d.stage;
+  const bool staged = n_waves > 1 && d.stage && !c->file;
   auto wave_width = [&](int w) {
     long long width = accesses_max - (long long)w * S;
     return (int)(width > S ? S : width);
   };
   MF_CUDA(cudaEventRecord(c->ev_fork[0], s));
   MF_CUDA(cudaStreamWaitEvent(c->side, c->ev_fork[0], 0));
+  if (c->file) MF_CUDA(enqueue_file_reads(c, layer, 0, false, c->side));  // wave 0's misses, file -> staging
   timer_mark(c, kTMaterialize, 0, c->side);
   MF_CUDA(launch_materialize(d, layer, 0, wave_width(0), c->side, nullptr, gemm));
   timer_mark(c, kTMaterialize, 1, c->side);
@@ -551,6 +584,7 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
       if (staged) {
         MF_CUDA(launch_stage_commit(d, layer, w, d.stage, c->side));
       } else {
+        if (c->file) MF_CUDA(enqueue_file_reads(c, layer, w, false, c->side));
         timer_mark(c, kTMaterialize, 0, c->side);
         MF_CUDA(launch_materialize(d, layer, w, width, c->side, nullptr, gemm));
         timer_mark(c, kTMaterialize, 1, c->side);
@@ -625,7 +659,7 @@ int mf_moe_forward_host(mf_ctx_t* c, int layer, const float* x, const float* rou
   // One token with pinned buffers: no copy steps.  The router reads x and the bias over the
   // CPU-GPU link (x once per block) and leaves a device copy of x for the FFN, which writes y
   // straight into the caller's buffer.
-  if (T == 1 && c->ffn_fused && !(((uintptr_t)x | (uintptr_t)router_w) & 15)) {
+  if (T == 1 && c->ffn_fused && !c->file && !(((uintptr_t)x | (uintptr_t)router_w) & 15)) {
     void *xd = nullptr, *bd = nullptr, *yd = nullptr;
     bool pinned = cudaHostGetDevicePointer(&xd, const_cast<float*>(x), 0) == cudaSuccess &&
                   cudaHostGetDevicePointer(&yd, y, 0) == cudaSuccess &&
@@ -774,11 +808,13 @@ int mf_check(mf_ctx_t* c) {
   MF_CUDA(cudaDeviceSynchronize());
   unsigned err = 0;
   MF_CUDA(cudaMemcpy(&err, c->d.err, sizeof(err), cudaMemcpyDeviceToHost));
-  if (err) {
-    MF_CUDA(cudaMemset(c->d.err, 0, sizeof(unsigned)));
-    return MF_E_TIMEOUT;
+  const int io = pack_file_error(c);
+  if (err) MF_CUDA(cudaMemset(c->d.err, 0, sizeof(unsigned)));
+  if (io) {
+    snprintf(g_cuda_err, sizeof(g_cuda_err), "split-pack file read: %s", strerror(io));
+    return MF_E_IO;
   }
-  return MF_OK;
+  return err ? MF_E_TIMEOUT : MF_OK;
 }
 
 void mf_destroy(mf_ctx_t* c) {

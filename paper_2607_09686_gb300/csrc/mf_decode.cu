@@ -417,7 +417,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ uint8_t* s_gu[kMaxTopK];  // each expert's HBM slot: gate/up region, down region
   __shared__ uint8_t* s_dn[kMaxTopK];
-  __shared__ const uint8_t* s_hgu[kMaxTopK];  // its payload in the pinned pack (missed experts)
+  __shared__ const uint8_t* s_hgu[kMaxTopK];  // its payload in host memory (missed experts)
   __shared__ float s_g[kMaxTopK];
   __shared__ int s_miss[kMaxTopK];
   __shared__ int s_gord[kMaxItemsF];  // the block's gate/up items: resident experts' first
@@ -458,7 +458,8 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
     s_gu[threadIdx.x] = slot;
     s_dn[threadIdx.x] = slot + d.lay.d_off;
-    s_hgu[threadIdx.x] = d.pack + ((size_t)layer * d.E + d.uniq[threadIdx.x]) * d.lay.stride;
+    s_hgu[threadIdx.x] = d.fstage ? d.fstage + (size_t)threadIdx.x * d.fstride  // staged from the file
+                                  : d.pack + ((size_t)layer * d.E + d.uniq[threadIdx.x]) * d.lay.stride;
     s_g[threadIdx.x] = d.g[threadIdx.x];
     s_miss[threadIdx.x] = d.umiss[threadIdx.x];
   }

@@ -41,7 +41,10 @@ struct Dev {
   int order;  // access order of calls with T > 1 (MF_ORDER_*)
   Layout lay;
   // memory
-  const uint8_t* pack;  // pinned host pack [L][E] slots, device-addressable
+  const uint8_t* pack;  // pinned host pack [L][E] slots, device-addressable (null for a file-backed pack)
+  const uint8_t* fstage;  // file-backed pack: pinned staging the host reads a call's misses into
+  uint64_t fstride;       // ... bytes per staged payload (a multiple of 4096); miss r of a one-token
+                          //     call (its rank r), or miss m of a wave, at fstage + index * fstride
   uint8_t* pool;        // HBM slot pool [L][S_alloc] slots
   // per-layer cache state
   int32_t* slot_of;    // [L][E]        expert -> slot or -1
@@ -209,12 +212,17 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
 
 }  // namespace mf
 
+namespace mf {
+struct PackFile;  // mf_packfile.cu
+}
+
 struct mf_ctx {
   mf_model_t model;
   mf_plan_t plan;
   int device;
   mf::Dev d;
-  uint8_t* pack_host;      // cudaHostAlloc'ed pack (host pointer)
+  uint8_t* pack_host;      // cudaHostAlloc'ed pack (host pointer; null for a file-backed pack)
+  mf::PackFile* file;      // the split-pack file of a file-backed context (else null)
   unsigned char* put_map;  // [L][E] which payloads have been put
   int64_t n_put;
   cudaStream_t side;       // materialisation stream
@@ -286,5 +294,12 @@ int prefill_tensor_maps(mf_ctx* c);  // encode tm_gu / tm_d for the context's po
 cudaError_t launch_tile_x(const Dev& d, const float* x, int T, cudaStream_t s);
 cudaError_t launch_prefill_gateup(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s);
 cudaError_t launch_prefill_down(const Dev& d, const CUtensorMap* tm, int layer, int wave, cudaStream_t s);
+// file-backed split-pack (mf_packfile.cu)
+int open_pack_file(mf_ctx* c, const char* path);  // MF_OK or an MF_E_* code
+void close_pack_file(mf_ctx* c);
+int pack_file_error(mf_ctx* c);  // errno of a failed read since the last call (0: none), cleared
+// a host function on `s` that reads the missed records of `layer` (one token: the call's misses
+// by rank; else wave `wave`'s misses in order) from the file into the staging
+cudaError_t enqueue_file_reads(mf_ctx* c, int layer, int wave, bool one_token, cudaStream_t s);
 
 }  // namespace mf

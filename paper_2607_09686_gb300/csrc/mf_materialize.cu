@@ -1,5 +1,7 @@
 // Materialisation of missed experts: pinned host pack -> HBM slot (section "Native Serving
-// Path": on a miss the runtime copies the requested expert block into an available slot).
+// Path": on a miss the runtime copies the requested expert block into an available slot).  With
+// a file-backed split-pack the host first reads the wave's misses from the file into pinned
+// staging (in miss order) and the same kernel copies them from there.
 //
 // The misses are decided on the device (slot resolve), so the copy is driven by the GPU
 // itself: SMs load 16-byte vectors straight from the pinned, device-mapped pack over the
@@ -36,7 +38,9 @@ __global__ void __launch_bounds__(kMatThreadsDense) k_materialize(Dev d, int lay
   const size_t step = (size_t)gridDim.x * blockDim.x * kUnroll;
   for (int m = 0; m < n_miss; ++m) {
     const int u = d.miss_list[wave * d.S_active + m];
-    const uint4* src = reinterpret_cast<const uint4*>(d.pack + ((size_t)layer * d.E + d.uniq[u]) * d.lay.stride);
+    const uint4* src = reinterpret_cast<const uint4*>(
+        d.fstage ? d.fstage + (size_t)m * d.fstride  // a file-backed pack: the host staged miss m here
+                 : d.pack + ((size_t)layer * d.E + d.uniq[u]) * d.lay.stride);
     uint4* dst = reinterpret_cast<uint4*>(dst_stage ? dst_stage + (size_t)m * d.lay.stride
                                                     : d.pool + ((size_t)layer * d.S_alloc + d.uslot[u]) * d.lay.stride);
     for (size_t i0 = (size_t)blockIdx.x * blockDim.x * kUnroll + threadIdx.x; i0 < nvec; i0 += step) {
