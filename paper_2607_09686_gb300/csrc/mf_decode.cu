@@ -24,6 +24,8 @@
 // deterministic and need no atomics.  Every wait is bounded; a wait that gives up sets the device error word
 // and the block stops.
 #include "mf_dequant.cuh"
+#include "mf_lru.cuh"
+#include "mf_route.cuh"
 
 namespace mf {
 namespace {
@@ -354,8 +356,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 // items through the ring, so the whole call's weights are in flight from the start.  The
 // consumers form h = silu(gate) * up for their gate/up items, publish it, meet every other block
 // at a grid-wide arrival counter (bounded wait), and then take the down items with the k experts'
-// h.  The counter never resets: each launch adds one arrival per block, and a block waits for the
-// multiple of gridDim.x that completes its launch.
+// h.  The counter never resets: each launch adds one arrival per block at each of its grid-wide
+// waits, and a block waits for the multiple of gridDim.x that completes the current one.
+//
+// With the routing inside (a one-token call whose router runs in the same launch, see
+// route_one_token), the blocks first compute the logits and meet at the counter once more before
+// the list of items is formed.
 //
 // Missed experts' bytes, by the whole warp: host_pull issues `bytes` (a multiple of 16) from the
 // pinned pack into shared memory as 16-byte cp.async pieces (every piece in flight at once; the
@@ -394,8 +400,10 @@ struct FusedCfg {
   uint32_t stage_bytes;  // gate/up item
   int red_floats;        // partial results: gate/up items x 16 warps, then k x rpc down rows
   uint32_t vq_bytes;
-  // shared memory: [NS gate/up stages | k down buffers | full | empty | full_d | red | vq]
-  size_t off_dn, off_bar, off_red, off_vq, total;
+  int route;  // 1: the launch routes the token itself (route_one_token)
+  int wpe;    // ... the router's warps per expert (router_warps_per_expert)
+  // shared memory: [NS gate/up stages | k down buffers | full | empty | full_d | red | vq | route]
+  size_t off_dn, off_bar, off_red, off_vq, off_route, total;
 };
 constexpr int kFusedBars = 2 * kMaxStages + kMaxTopK;
 
@@ -410,9 +418,239 @@ __device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, uns
   return false;
 }
 
+// ---- routing of a one-token call inside the fused kernel
+// Block b computes the logits of experts b, b + gridDim.x, ... and stores them, each with the
+// router's arithmetic in the router's order (the router's wpe warps of an expert become threads
+// 0 .. 32 wpe - 1 here: thread part * 32 + lane sums the float4 columns part * 32 + lane +
+// i * 32 wpe in increasing i, the warps' pairs are added lane-wise by the same butterfly and the
+// parts in order), so the logits, and everything that follows, are the router's bits; after a grid-wide
+// arrival on the kernel's counter every block reads all E logits, ranks them and takes the
+// softmax over the chosen exactly as the router does (rank_topk, topk_softmax), and replays the
+// layer's least-recently-used replacement (lru_warp: the router's decisions) on its own copy of
+// the cache state, requested before the logits.  So every block knows each chosen expert's slot
+// and whether it missed -- a resident expert that an earlier miss of the same call evicts
+// included -- without waiting for another block.  Block 0 alone writes the call's records: idx
+// and g, the access record and counters, and the layer's new cache state.
+struct RouteSmem {
+  uint64_t* last;  // [S_alloc] the layer's cache state, replayed by this block
+  float* z;        // [E] logits
+  int* slot_of;    // [E]
+  int* expert_of;  // [S_alloc]
+  float* ps;       // [kThreadsF / 32] each warp's compensated partial
+  float* pc;
+  int* sel;    // [kMaxTopK] chosen experts in rank order
+  float* zsel; // [kMaxTopK] their logits
+  float* g;    // [kMaxTopK] their router weights
+  int* uslot;  // [kMaxTopK] their slots after the replacement
+  int* umiss;  // [kMaxTopK] 1 where the access missed
+  int* ok;     // [1] the grid-wide arrival completed in time
+};
+constexpr int kWarpsF = kThreadsF / 32;
+size_t route_bytes(int E, int S) {
+  return (size_t)8 * S + 8 * (size_t)E + 4 * (size_t)S + 8 * kWarpsF + 20 * kMaxTopK + 16;
+}
+__device__ __forceinline__ RouteSmem route_smem(unsigned char* p, int E, int S) {
+  RouteSmem r;
+  r.last = reinterpret_cast<uint64_t*>(p);
+  r.z = reinterpret_cast<float*>(p + (size_t)8 * S);
+  r.slot_of = reinterpret_cast<int*>(r.z + E);
+  r.expert_of = r.slot_of + E;
+  r.ps = reinterpret_cast<float*>(r.expert_of + S);
+  r.pc = r.ps + kWarpsF;
+  r.sel = reinterpret_cast<int*>(r.pc + kWarpsF);
+  r.zsel = reinterpret_cast<float*>(r.sel + kMaxTopK);
+  r.g = r.zsel + kMaxTopK;
+  r.uslot = reinterpret_cast<int*>(r.g + kMaxTopK);
+  r.umiss = r.uslot + kMaxTopK;
+  r.ok = r.umiss + kMaxTopK;
+  return r;
+}
+constexpr int kPreF = (kMaxExperts + kThreadsF - 1) / kThreadsF;  // state entries a thread requests
+constexpr int kRouteChunk = 4;  // float4 loads of W_r (and of x) a thread issues before using them
+
+// Every thread of the block calls it (block barriers inside), right after the kernel's wait for
+// the previous launch; it arrives once at the grid-wide counter.
+__device__ __forceinline__ void route_one_token(const Dev& d, int layer, const float* __restrict__ x,
+                                                const float* __restrict__ wr, const float* __restrict__ bias,
+                                                int wpe, const RouteSmem& r) {
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int E = d.E, S = d.S_active, k = d.k, n4 = d.H / 4;
+  int32_t* g_slot_of = d.slot_of + (size_t)layer * E;
+  int32_t* g_expert_of = d.expert_of + (size_t)layer * d.S_alloc;
+  uint64_t* g_last = d.last_use + (size_t)layer * d.S_alloc;
+  int pre_slot[kPreF], pre_exp[kPreF];
+  uint64_t pre_last[kPreF];
+#pragma unroll
+  for (int i = 0; i < kPreF; ++i) {
+    const int e = tid + i * kThreadsF;
+    pre_slot[i] = e < E ? g_slot_of[e] : -1;
+    pre_exp[i] = e < S ? g_expert_of[e] : -1;
+    pre_last[i] = e < S ? g_last[e] : 0;
+  }
+  const uint64_t clock0 = warp == 0 ? d.clock[layer] : 0;
+  const uint64_t pol = l2_evict_last();  // W_r is read again by the layer's next call
+  const float4* x4 = reinterpret_cast<const float4*>(x);
+  const int step = wpe * 32;
+  for (int e = blockIdx.x; e < E; e += gridDim.x) {  // block-uniform
+    const float4* w4 = reinterpret_cast<const float4*>(wr + (size_t)e * d.H);
+    float s = 0.f, c = 0.f;
+    if (tid < step)
+      for (int q0 = tid; q0 < n4; q0 += kRouteChunk * step) {
+        float4 a[kRouteChunk], b[kRouteChunk];
+#pragma unroll
+        for (int u = 0; u < kRouteChunk; ++u) {  // the chunk's loads first
+          const int q = q0 + u * step;
+          if (q < n4) {
+            a[u] = ld_hint(w4 + q, pol);
+            b[u] = __ldg(x4 + q);
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kRouteChunk; ++u)
+          if (q0 + u * step < n4) {
+            dot2(s, c, a[u].x, b[u].x);
+            dot2(s, c, a[u].y, b[u].y);
+            dot2(s, c, a[u].z, b[u].z);
+            dot2(s, c, a[u].w, b[u].w);
+          }
+      }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      const float so = __shfl_xor_sync(0xffffffffu, s, off);
+      const float co = __shfl_xor_sync(0xffffffffu, c, off);
+      pair_add(s, c, so, co);
+    }
+    if (lane == 0 && warp < wpe) {
+      r.ps[warp] = s;
+      r.pc[warp] = c;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      float zs = r.ps[0], zc = r.pc[0];
+      for (int w = 1; w < wpe; ++w) pair_add(zs, zc, r.ps[w], r.pc[w]);
+      float z = __fadd_rn(zs, zc);
+      if (bias) z = __fadd_rn(z, bias[e]);
+      d.zlog[e] = z;
+    }
+    __syncthreads();  // the partials are reused by the block's next expert
+  }
+  // this block's logits were stored by thread 0, before its (release) arrival
+  if (tid == 0) r.ok[0] = grid_arrive_wait(d.work, d.err, d.wait_ns) ? 1 : 0;
+#pragma unroll
+  for (int i = 0; i < kPreF; ++i) {  // the cache state (landed meanwhile) into shared memory
+    const int e = tid + i * kThreadsF;
+    if (e < E) r.slot_of[e] = pre_slot[i];
+    if (e < S) {
+      r.expert_of[e] = pre_exp[i];
+      r.last[e] = pre_last[i];
+    }
+  }
+  __syncthreads();
+  for (int e = tid; e < E; e += kThreadsF) r.z[e] = __ldcg(d.zlog + e);  // other blocks wrote them
+  rank_topk(r.z, E, k, r.sel, r.zsel);                                  // (block barrier first)
+  if (warp == 0) {
+    const bool pub = blockIdx.x == 0;
+    const float g = topk_softmax(r.zsel, k);
+    if (lane < k) r.g[lane] = g;
+    if (pub && lane < k) {
+      d.idx[lane] = r.sel[lane];
+      d.g[lane] = g;
+    }
+    if (pub && lane == 0) d.info[2] = 0;
+    __syncwarp();
+    // one token: the k chosen experts are distinct, the accesses are them in rank order
+    lru_warp(d, layer, k, r.sel, r.slot_of, r.expert_of, r.last, r.uslot, __shfl_sync(0xffffffffu, clock0, 0), pub,
+             r.umiss);
+    if (pub) {
+      if (lane < k) {  // one assignment per distinct expert: t = 0, j = u
+        d.pos_slot[lane] = r.uslot[lane];
+        d.asg[lane] = lane;
+        d.asg_off[lane] = lane;
+      }
+      if (lane == 0) d.asg_off[k] = k;
+      for (int e = lane; e < E; e += 32) g_slot_of[e] = r.slot_of[e];
+      for (int q = lane; q < S; q += 32) {
+        g_expert_of[q] = r.expert_of[q];
+        g_last[q] = r.last[q];
+      }
+    }
+  }
+  __syncthreads();
+}
+
+// ---- x split by the consumers, kG = kW / 4 threads (consecutive lanes) per group of x, each
+// thread one word of four values; kXR rounds of 512 words (the fused path takes H <= 4096).
+// The same pieces as quant_vals of the whole group: the group's largest magnitude m by shuffles,
+// each value scaled by 2^-e_g (e_g: m's exponent) and split by 127 / (m 2^-e_g), the piece sums
+// added over the kG threads; then the vector's exponent and rescale_group as in split_vectors.
+constexpr int kXR = 2;
+template <int QT>
+__device__ __forceinline__ void split_x_words(const float4 (&xv)[kXR], int n_words, XQ<QT>* dst, int* s_max,
+                                              int* s_exp) {
+  constexpr int kG = Vec<QT>::kW / 4;
+  int eg[kXR];
+#pragma unroll
+  for (int rr = 0; rr < kXR; ++rr) {
+    const int w = (int)threadIdx.x + rr * kConsumers * 32, gi = w / kG, part = w % kG;
+    const float4 v = xv[rr];
+    float m = fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
+#pragma unroll
+    for (int o = 1; o < kG; o <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    eg[rr] = group_exponent(m);
+    const int ne = eg[rr] == kNoExp ? 0 : -eg[rr];
+    const float sa = pow2i(ne / 2), sb = pow2i(ne - ne / 2);
+    const float ms = m * sa * sb;  // exact: the largest value scaled by a power of two
+    const float inv = ms > 0x1p-100f ? 127.f / ms : 0.f;
+    const float vv[4] = {v.x * sa * sb, v.y * sa * sb, v.z * sa * sb, v.w * sa * sb};
+    uint32_t b1 = 0, b2 = 0, b3 = 0;
+    int s1 = 0, s2 = 0, s3 = 0;
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      const float t = vv[jj] * inv;
+      const int a = __float2int_rn(t);
+      const float e = (t - (float)a) * 127.f;
+      const int b = __float2int_rn(e);
+      const int c = __float2int_rn((e - (float)b) * 127.f);
+      s1 += a;
+      s2 += b;
+      s3 += c;
+      b1 |= (uint32_t)(a & 0xFF) << (8 * jj);
+      b2 |= (uint32_t)(b & 0xFF) << (8 * jj);
+      b3 |= (uint32_t)(c & 0xFF) << (8 * jj);
+    }
+#pragma unroll
+    for (int o = 1; o < kG; o <<= 1) {
+      s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+      s3 += __shfl_xor_sync(0xffffffffu, s3, o);
+    }
+    if (w < n_words) {
+      dst[gi].p1[part] = b1;
+      dst[gi].p2[part] = b2;
+      dst[gi].p3[part] = b3;
+      if (part == 0) {
+        constexpr int off = QT == kQ8 ? 128 : 8;
+        dst[gi].k12 = off * (s1 * 127 + s2);
+        dst[gi].k3 = off * s3;
+        dst[gi].sf = inv > 0.f ? ms / 127.f / 16129.f : 0.f;
+        atomicMax(s_max, eg[rr]);
+      }
+    }
+  }
+  named_bar_sync(1, kConsumers * 32);
+#pragma unroll
+  for (int rr = 0; rr < kXR; ++rr) {
+    const int w = (int)threadIdx.x + rr * kConsumers * 32;
+    if (w < n_words && w % kG == 0) rescale_group<QT>(dst[w / kG], eg[rr], vector_exponent(*s_max));
+  }
+  if (threadIdx.x == 0) *s_exp = vector_exponent(*s_max);
+  named_bar_sync(1, kConsumers * 32);
+}
+
 template <int QT, int VPL, int VPLD>
 __global__ void __launch_bounds__(kThreadsF, 1)
-    k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, float* __restrict__ y, FusedCfg f) {
+    k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, const float* __restrict__ wr,
+               const float* __restrict__ bias, float* __restrict__ y, FusedCfg f) {
   constexpr int kW = Vec<QT>::kW;
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ uint8_t* s_gu[kMaxTopK];  // each expert's HBM slot: gate/up region, down region
@@ -450,11 +688,29 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     s_xmax = kNoExp;
   }
   if (threadIdx.x < kMaxTopK) s_hmax[threadIdx.x] = kNoExp;
-  pdl_wait();  // the router's outputs (and the caller's x) are complete and visible
-  float xv[kW];  // consumer thread i < n_vec: group i of x, requested while the block sets up
-  const bool x_mine = warp < kConsumers && (int)threadIdx.x < cg.n_vec;
-  if (x_mine) load_group<QT>(x + (size_t)threadIdx.x * kW, xv);
-  if (threadIdx.x < k) {  // one token: access u = rank j
+  pdl_wait();  // the previous launch (the router, or the previous call) is complete and visible
+  // consumer thread t: words t, t + 512 of x (four values each), requested while the block sets up
+  const int n_xw = d.H / 4;
+  float4 xv[kXR];
+#pragma unroll
+  for (int rr = 0; rr < kXR; ++rr) {
+    const int w = (int)threadIdx.x + rr * kConsumers * 32;
+    xv[rr] = warp < kConsumers && w < n_xw ? __ldg(reinterpret_cast<const float4*>(x) + w)
+                                           : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  if (f.route) {  // the token's routing and slot replacement, in this launch
+    const RouteSmem r = route_smem(smem + f.off_route, d.E, d.S_alloc);
+    route_one_token(d, layer, x, wr, bias, f.wpe, r);
+    if (threadIdx.x < k) {
+      const int j = threadIdx.x;
+      uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + r.uslot[j]) * d.lay.stride;
+      s_gu[j] = slot;
+      s_dn[j] = slot + d.lay.d_off;
+      s_hgu[j] = d.pack + ((size_t)layer * d.E + r.sel[j]) * d.lay.stride;
+      s_g[j] = r.g[j];
+      s_miss[j] = r.umiss[j];
+    }
+  } else if (threadIdx.x < k) {  // one token, routed by the router: access u = rank j
     uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
     s_gu[threadIdx.x] = slot;
     s_dn[threadIdx.x] = slot + d.lay.d_off;
@@ -603,18 +859,8 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       const int nv = (d.lay.qrow_gu / 16) / cs;
       const int v0 = col * nv;
       const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-      {  // x split into int8 pieces, scaled by the power of two of its largest magnitude
-        XQ<QT>* dst = reinterpret_cast<XQ<QT>*>(sm.vq);
-        const int eg = x_mine ? group_exponent(group_absmax<QT>(xv)) : kNoExp;
-        if (x_mine) {
-          dst[threadIdx.x] = quant_vals<QT>(xv, eg == kNoExp ? 0 : -eg);
-          atomicMax(&s_xmax, eg);
-        }
-        named_bar_sync(1, kConsumers * 32);
-        if (x_mine) rescale_group<QT>(dst[threadIdx.x], eg, vector_exponent(s_xmax));
-        if (threadIdx.x == 0) s_xexp = vector_exponent(s_xmax);
-        named_bar_sync(1, kConsumers * 32);
-      }
+      // x split into int8 pieces, scaled by the power of two of its largest magnitude
+      split_x_words<QT>(xv, n_xw, reinterpret_cast<XQ<QT>*>(sm.vq), &s_xmax, &s_xexp);
       XQ<QT> xr[VPL];
 #pragma unroll
       for (int i = 0; i < VPL; ++i) {
@@ -834,8 +1080,10 @@ cudaError_t down_pipe_q(const Dev& d, int layer, float* y, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-FusedCfg fused_cfg(const Dev& d) {
+FusedCfg fused_cfg(const Dev& d, bool route) {
   FusedCfg f;
+  f.route = route ? 1 : 0;
+  f.wpe = route ? router_warps_per_expert(d.E, d.H) : 0;
   f.g = gateup_cfg(d);
   f.rpc = (d.H + sm_count() - 1) / sm_count();
   f.dn_bytes = (uint32_t)f.rpc * d.lay.rs_d;
@@ -844,8 +1092,9 @@ FusedCfg fused_cfg(const Dev& d) {
   f.stage_bytes = f.g.stage_bytes;
   f.red_floats = f.g.max_mine * kConsumers + d.k * f.rpc;
   f.vq_bytes = f.g.vq_bytes > hv_bytes ? f.g.vq_bytes : hv_bytes;
+  const size_t rbytes = route ? route_bytes(d.E, d.S_alloc) : 0;
   const size_t fixed = (size_t)d.k * f.dn_bytes + kFusedBars * sizeof(uint64_t) +
-                       (size_t)f.red_floats * sizeof(float) + f.vq_bytes;
+                       (size_t)f.red_floats * sizeof(float) + f.vq_bytes + 16 + rbytes;
   const size_t budget = kFusedSmem - 1024;  // - the kernel's static shared memory
   const size_t ns = fixed < budget ? (budget - fixed) / f.stage_bytes : 0;
   f.NS = (int)(ns > (size_t)kMaxStages ? kMaxStages : ns);
@@ -853,19 +1102,20 @@ FusedCfg fused_cfg(const Dev& d) {
   f.off_bar = f.off_dn + (size_t)d.k * f.dn_bytes;
   f.off_red = f.off_bar + kFusedBars * sizeof(uint64_t);
   f.off_vq = f.off_red + (((size_t)f.red_floats * sizeof(float) + 15) & ~(size_t)15);
-  f.total = f.off_vq + f.vq_bytes;
+  f.off_route = (f.off_vq + f.vq_bytes + 15) & ~(size_t)15;
+  f.total = f.off_route + rbytes;
   return f;
 }
 
 size_t fused_smem(const FusedCfg& f) { return f.total; }
 
-// One block per SM.  The launch is programmatic (it may begin while the router finishes: the
-// kernel's prologue touches only shared memory and it waits for the router before reading
-// anything else); where the driver refuses that, a cooperative launch.  Blocks wait for each
-// other only through bounded waits.
+// One block per SM.  The launch is programmatic (it may begin while the previous kernel of the
+// stream finishes: the kernel's prologue touches only shared memory and it waits for that kernel
+// before reading anything else); where the driver refuses that, a cooperative launch.  Blocks
+// wait for each other only through bounded waits.
 template <class Kern>
-cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x, float* y,
-                       const FusedCfg& f) {
+cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x,
+                       const float* wr, const float* bias, float* y, const FusedCfg& f) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -880,23 +1130,24 @@ cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int
   if (pdl_ok) {
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    e = cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
+    e = cudaLaunchKernelEx(&cfg, kern, d, layer, x, wr, bias, y, f);
     if (e == cudaSuccess) return e;
     cudaGetLastError();
     pdl_ok = false;
   }
   attr[0].id = cudaLaunchAttributeCooperative;  // every block resident: they wait for each other
   attr[0].val.cooperative = 1;
-  return cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
+  return cudaLaunchKernelEx(&cfg, kern, d, layer, x, wr, bias, y, f);
 }
 
 template <int QT>
-cudaError_t ffn_pipe_q(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
-  const FusedCfg f = fused_cfg(d);
+cudaError_t ffn_pipe_q(const Dev& d, int layer, const float* x, const float* wr, const float* bias, float* y,
+                       cudaStream_t s) {
+  const FusedCfg f = fused_cfg(d, wr != nullptr);
   const size_t smem = fused_smem(f);
   const int vx = vpl_for((d.lay.qrow_gu / 16) / f.g.cs), vh = vpl_for(d.lay.qrow_d / 16);
 #define MF_FF(A, B) \
-  if (vx == A && vh == B) return launch_ffn(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, y, f);
+  if (vx == A && vh == B) return launch_ffn(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, wr, bias, y, f);
   MF_FF(1, 1) MF_FF(1, 2) MF_FF(2, 1) MF_FF(2, 2)
   if constexpr (QT == kQ8) {  // Q4_0 takes at most two vectors per lane (decode_pipe_ok)
     MF_FF(1, 3) MF_FF(2, 3) MF_FF(3, 1) MF_FF(3, 2) MF_FF(3, 3) MF_FF(4, 1) MF_FF(4, 2) MF_FF(4, 3)
@@ -931,12 +1182,23 @@ cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStrea
 size_t decode_smem_bytes(const Dev& d, int which) { return smem_bytes(which == 0 ? gateup_cfg(d) : down_cfg(d)); }
 
 bool ffn_fused_ok(const Dev& d) {
-  const FusedCfg f = fused_cfg(d);
-  return decode_pipe_ok(d) && f.NS >= 4 && f.g.max_mine <= kMaxItemsF;
+  const FusedCfg f = fused_cfg(d, false);
+  return decode_pipe_ok(d) && f.NS >= 4 && f.g.max_mine <= kMaxItemsF && d.H / 4 <= kXR * kConsumers * 32;
+}
+
+bool ffn_routed_ok(const Dev& d) {
+  return ffn_fused_ok(d) && fused_cfg(d, true).NS >= 4 && d.E <= kMaxExperts;
 }
 
 cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
-  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, y, s) : ffn_pipe_q<kQ4>(d, layer, x, y, s);
+  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, nullptr, nullptr, y, s)
+                            : ffn_pipe_q<kQ4>(d, layer, x, nullptr, nullptr, y, s);
+}
+
+cudaError_t launch_ffn_routed(const Dev& d, int layer, const float* x, const float* wr, const float* bias, float* y,
+                              cudaStream_t s) {
+  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, wr, bias, y, s)
+                            : ffn_pipe_q<kQ4>(d, layer, x, wr, bias, y, s);
 }
 
 }  // namespace mf

@@ -59,6 +59,7 @@ struct Dev {
   uint8_t* tr_hit;     // [L][E]
   // per-call scratch
   float2* zpart;       // router, T >= kTiledMinT: compensated logit pairs [K split][T][E]
+  float* zlog;         // [E]           logits of a one-token call routed inside the fused kernel
   int32_t* idx;        // [T_max][k]
   float* g;            // [T_max][k]
   int32_t* uniq;       // [E]           distinct experts in access order
@@ -244,6 +245,7 @@ struct mf_ctx {
   uint64_t overhead_bytes;
   bool decode_pipe;  // batch-1 calls use the pipelined decode kernels
   bool ffn_fused;    // ... fused into one cooperative launch
+  bool ffn_routed;   // ... with the token's routing inside that launch (device x, pinned pack)
   int prefill_min_t;  // calls with T >= this use the tensor-core grouped GEMMs (0 = never)
   uint8_t* gemm_scratch;  // x and h tiles of the tensor-core path (allocated when first enabled)
   bool tmaps_ok;
@@ -285,6 +287,13 @@ bool decode_pipe_ok(const Dev& d);
 // both projections of one token in one cooperative launch (d.work holds its arrival counter)
 bool ffn_fused_ok(const Dev& d);
 cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s);
+// one-token call, routed inside the fused kernel (router, slot replacement and expert FFN in one
+// launch), with the one-token router's arithmetic order
+int router_cluster_size(int H);
+int router_warps_per_expert(int E, int H);
+bool ffn_routed_ok(const Dev& d);
+cudaError_t launch_ffn_routed(const Dev& d, int layer, const float* x, const float* wr, const float* bias, float* y,
+                              cudaStream_t s);
 // many tokens per expert: tcgen05 grouped GEMMs (gate/up + SwiGLU, down) per wave
 constexpr int kPrefillMinTokens = 256;
 bool prefill_shape_ok(int hidden, int inter);
