@@ -86,7 +86,7 @@ struct Carve {
 
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
-  uint64_t zpart, zlog, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
+  uint64_t zpart, ztag, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
   uint64_t work, err, tb_off, sx, sb, sy, sidx, sw, stage;
   uint64_t total;
 };
@@ -105,7 +105,7 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.tr_slot = c.take<int32_t>(L * E);
   o.tr_hit = c.take<uint8_t>(L * E);
   o.zpart = c.take<float2>(router_part_pairs(Tm, (int)E, (int)H));
-  o.zlog = c.take<float>(E);
+  o.ztag = c.take<uint64_t>(E);
   o.idx = c.take<int32_t>((uint64_t)Tm * k);
   o.g = c.take<float>((uint64_t)Tm * k);
   o.uniq = c.take<int32_t>(E);
@@ -345,7 +345,7 @@ int create_ctx(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devi
   d.tr_slot = reinterpret_cast<int32_t*>(base + so.tr_slot);
   d.tr_hit = reinterpret_cast<uint8_t*>(base + so.tr_hit);
   d.zpart = reinterpret_cast<float2*>(base + so.zpart);
-  d.zlog = reinterpret_cast<float*>(base + so.zlog);
+  d.ztag = reinterpret_cast<unsigned long long*>(base + so.ztag);
   d.idx = reinterpret_cast<int32_t*>(base + so.idx);
   d.g = reinterpret_cast<float*>(base + so.g);
   d.uniq = reinterpret_cast<int32_t*>(base + so.uniq);

@@ -59,11 +59,21 @@ __device__ __forceinline__ void rank_topk(const float* s_z, int E, int k, int* s
     const bool valid = e < E;
     const float z = valid ? s_z[e] : 0.f;
     int r = 0;
-    if (valid)
-      for (int e2 = part; e2 < E; e2 += tpe) {
+    if (valid) {
+      int e2 = part;
+      for (; e2 + 7 * tpe < E; e2 += 8 * tpe) {  // eight loads in flight
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int ee = e2 + u * tpe;
+          const float z2 = s_z[ee];
+          r += (z2 > z) || (z2 == z && ee < e);
+        }
+      }
+      for (; e2 < E; e2 += tpe) {
         const float z2 = s_z[e2];
         r += (z2 > z) || (z2 == z && e2 < e);
       }
+    }
     for (int off = tpe >> 1; off > 0; off >>= 1) r += __shfl_xor_sync(0xffffffffu, r, off);
     if (valid && part == 0 && r < k) {
       s_sel[r] = e;
