@@ -86,7 +86,7 @@ struct Carve {
 
 struct ScratchOffsets {
   uint64_t slot_of, expert_of, last_use, clock, stats, tr_n, tr_expert, tr_slot, tr_hit;
-  uint64_t zpart, ztag, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
+  uint64_t zpart, idx, g, uniq, uslot, umiss, asg_off, asg, pos_slot, info, miss_list, h, part;
   uint64_t work, err, tb_off, sx, sb, sy, sidx, sw, stage;
   uint64_t total;
 };
@@ -105,7 +105,6 @@ ScratchOffsets scratch_layout(const mf_model_t& m, int S, int Tm) {
   o.tr_slot = c.take<int32_t>(L * E);
   o.tr_hit = c.take<uint8_t>(L * E);
   o.zpart = c.take<float2>(router_part_pairs(Tm, (int)E, (int)H));
-  o.ztag = c.take<uint64_t>(E);
   o.idx = c.take<int32_t>((uint64_t)Tm * k);
   o.g = c.take<float>((uint64_t)Tm * k);
   o.uniq = c.take<int32_t>(E);
@@ -345,7 +344,6 @@ int create_ctx(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devi
   d.tr_slot = reinterpret_cast<int32_t*>(base + so.tr_slot);
   d.tr_hit = reinterpret_cast<uint8_t*>(base + so.tr_hit);
   d.zpart = reinterpret_cast<float2*>(base + so.zpart);
-  d.ztag = reinterpret_cast<unsigned long long*>(base + so.ztag);
   d.idx = reinterpret_cast<int32_t*>(base + so.idx);
   d.g = reinterpret_cast<float*>(base + so.g);
   d.uniq = reinterpret_cast<int32_t*>(base + so.uniq);
@@ -402,7 +400,6 @@ int create_ctx(mf_ctx_t** out, const mf_model_t* m, const mf_plan_t* p, int devi
   }
   c->decode_pipe = decode_pipe_ok(d) && getenv("MF_DECODE_SIMPLE") == nullptr;
   c->ffn_fused = c->decode_pipe && ffn_fused_ok(d) && getenv("MF_DECODE_UNFUSED") == nullptr;
-  c->ffn_routed = c->ffn_fused && ffn_routed_ok(d) && getenv("MF_DECODE_ROUTER") == nullptr;
   c->tmaps_ok = prefill_shape_ok(d.H, d.I) && prefill_tensor_maps(c) == 0;
   c->prefill_min_t = 0;
   if (c->tmaps_ok && gemm_at_create(*m, Tm)) {
@@ -532,14 +529,6 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
   const Dev& d = c->d;
   const int S = d.S_active;
 
-  if (T == 1 && c->ffn_routed && !c->file) {  // one launch: routing, slot replacement, misses, expert FFN
-    timer_mark(c, kTFfn, 0, s);
-    MF_CUDA(launch_ffn_routed(d, layer, x, router_w, logit_bias, y, s));
-    timer_mark(c, kTFfn, 1, s);
-    if (idx_out) MF_CUDA(cudaMemcpyAsync(idx_out, d.idx, sizeof(int32_t) * d.k, cudaMemcpyDeviceToDevice, s));
-    if (w_out) MF_CUDA(cudaMemcpyAsync(w_out, d.g, sizeof(float) * d.k, cudaMemcpyDeviceToDevice, s));
-    return MF_OK;
-  }
   timer_mark(c, kTRouter, 0, s);
   MF_CUDA(launch_router(d, x, router_w, logit_bias, T, layer, s));
   timer_mark(c, kTRouter, 1, s);
@@ -551,7 +540,7 @@ int mf_moe_forward(mf_ctx_t* c, int layer, const float* x, const float* router_w
 
   const bool gemm = T > 1 && c->prefill_min_t > 0 && T >= c->prefill_min_t;
 
-  if (T == 1 && c->ffn_fused) {  // router, then one launch: expert FFN, with the misses materialised inside
+  if (T == 1 && c->ffn_fused) {  // one launch: expert FFN, with the misses materialised inside
     if (c->file) MF_CUDA(enqueue_file_reads(c, layer, 0, true, s));  // the misses, file -> staging
     timer_mark(c, kTFfn, 0, s);
     MF_CUDA(launch_ffn_single(d, layer, x, y, s));

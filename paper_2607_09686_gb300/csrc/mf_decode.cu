@@ -24,8 +24,6 @@
 // deterministic and need no atomics.  Every wait is bounded; a wait that gives up sets the device error word
 // and the block stops.
 #include "mf_dequant.cuh"
-#include "mf_lru.cuh"
-#include "mf_route.cuh"
 
 namespace mf {
 namespace {
@@ -97,20 +95,7 @@ __device__ __forceinline__ void split_vectors(const float* __restrict__ src, int
       load_group<QT, kCoherent>(src + (size_t)i * kW, v);
       eg[q] = group_exponent(group_absmax<QT>(v));
       dst[i] = quant_vals<QT>(v, eg[q] == kNoExp ? 0 : -eg[q]);
-    }
-    // the vector's largest exponent: one shared atomic per warp where its groups share a vector
-    const int i_w = i0 - (i0 & 31) + q * nt;  // the warp's first group
-    if (i_w < n) {
-      const int rv = i < n ? i / per : -1;
-      const int e = i < n ? eg[q] : kNoExp;
-      if (__all_sync(0xffffffffu, i >= n || rv == i_w / per)) {
-        int wm = e;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) wm = max(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-        if ((i0 & 31) == 0 && wm != kNoExp) atomicMax(&s_max[i_w / per], wm);
-      } else if (i < n) {
-        atomicMax(&s_max[rv], e);
-      }
+      atomicMax(&s_max[i / per], eg[q]);
     }
   }
   named_bar_sync(1, nt);
@@ -369,12 +354,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_down_pipe(Dev d, int layer, flo
 // items through the ring, so the whole call's weights are in flight from the start.  The
 // consumers form h = silu(gate) * up for their gate/up items, publish it, meet every other block
 // at a grid-wide arrival counter (bounded wait), and then take the down items with the k experts'
-// h.  The counter never resets: each launch adds one arrival per block at each of its grid-wide
-// waits, and a block waits for the multiple of gridDim.x that completes the current one.
-//
-// With the routing inside (a one-token call whose router runs in the same launch, see
-// route_one_token), the blocks first compute the logits and meet at the counter once more before
-// the list of items is formed.
+// h.  The counter never resets: each launch adds one arrival per block, and a block waits for the
+// multiple of gridDim.x that completes its launch.
 //
 // Missed experts' bytes, by the whole warp: host_pull issues `bytes` (a multiple of 16) from the
 // pinned pack into shared memory as 16-byte cp.async pieces (every piece in flight at once; the
@@ -413,12 +394,10 @@ struct FusedCfg {
   uint32_t stage_bytes;  // gate/up item
   int red_floats;        // partial results: gate/up items x 16 warps, then k x rpc down rows
   uint32_t vq_bytes;
-  int route;  // 1: the launch routes the token itself (route_one_token)
-  int wpe;    // ... the router's warps per expert (router_warps_per_expert)
-  // shared memory: [NS gate/up stages | k down buffers | full | empty | full_d | red | vq | route]
-  size_t off_dn, off_bar, off_red, off_vq, off_route, total;
+  // shared memory: [NS gate/up stages | k down buffers | full | empty | full_d | red | vq]
+  size_t off_dn, off_bar, off_red, off_vq, total;
 };
-constexpr int kFusedBars = 2 * kMaxStages + kMaxTopK + 1;  // + x staged (routed launches)
+constexpr int kFusedBars = 2 * kMaxStages + kMaxTopK;
 
 // The arrival is a release (the block's h, written before it and published to this thread by the
 // block barrier, becomes visible with it); the polling loads acquire.  Bounded in time.
@@ -431,284 +410,9 @@ __device__ __forceinline__ bool grid_arrive_wait(unsigned long long* arrive, uns
   return false;
 }
 
-// ---- routing of a one-token call inside the fused kernel
-// Block b computes the logits of experts b, b + gridDim.x, ... and stores them, each with the
-// router's arithmetic in the router's order (the router's wpe warps of an expert become threads
-// 0 .. 32 wpe - 1 here: thread part * 32 + lane sums the float4 columns part * 32 + lane +
-// i * 32 wpe in increasing i, the warps' pairs are added lane-wise by the same butterfly and the
-// parts in order), so the logits, and everything that follows, are the router's bits.  A logit
-// is stored together with the call's epoch in one 64-bit word (tagged), so a block that reads all
-// E of them waits for exactly those words, with no grid-wide barrier and no fence.  Every block
-// then ranks the logits and takes the softmax over the chosen as the router does (rank_topk,
-// topk_softmax).  When every chosen expert is resident nothing is placed or evicted: the slots are
-// the resident ones, and block 0's link warp (idle in such a call) does the replacement's
-// bookkeeping later.  Otherwise every block replays the layer's least-recently-used replacement
-// (lru_warp: the router's decisions) on its own copy of the cache state, requested before the
-// logits, so it knows each chosen expert's slot and whether it missed -- a resident expert that
-// an earlier miss of the same call evicts included -- without waiting for another block.  Block 0
-// alone writes the call's records: idx and g, the access record and counters, and the layer's
-// new cache state.
-struct RouteSmem {
-  uint64_t* last;  // [S_alloc] the layer's cache state, replayed by this block
-  float* z;        // [E] logits
-  int* slot_of;    // [E]
-  int* expert_of;  // [S_alloc]
-  float* ps;       // [kThreadsF / 32] each warp's compensated partial
-  float* pc;
-  int* sel;    // [kMaxTopK] chosen experts in rank order
-  float* zsel; // [kMaxTopK] their logits
-  float* g;    // [kMaxTopK] their router weights
-  int* uslot;  // [kMaxTopK] their slots after the replacement
-  int* umiss;  // [kMaxTopK] 1 where the access missed
-  int* later;  // [1] block 0: the replacement's bookkeeping is left to the link warp (every access hit)
-};
-constexpr int kWarpsF = kThreadsF / 32;
-size_t route_bytes(int E, int S) {
-  return (size_t)8 * S + 8 * (size_t)E + 4 * (size_t)S + 8 * kWarpsF + 20 * kMaxTopK + 16;
-}
-__device__ __forceinline__ RouteSmem route_smem(unsigned char* p, int E, int S) {
-  RouteSmem r;
-  r.last = reinterpret_cast<uint64_t*>(p);
-  r.z = reinterpret_cast<float*>(p + (size_t)8 * S);
-  r.slot_of = reinterpret_cast<int*>(r.z + E);
-  r.expert_of = r.slot_of + E;
-  r.ps = reinterpret_cast<float*>(r.expert_of + S);
-  r.pc = r.ps + kWarpsF;
-  r.sel = reinterpret_cast<int*>(r.pc + kWarpsF);
-  r.zsel = reinterpret_cast<float*>(r.sel + kMaxTopK);
-  r.g = r.zsel + kMaxTopK;
-  r.uslot = reinterpret_cast<int*>(r.g + kMaxTopK);
-  r.umiss = r.uslot + kMaxTopK;
-  r.later = r.umiss + kMaxTopK;
-  return r;
-}
-constexpr int kPreF = (kMaxExperts + kThreadsF - 1) / kThreadsF;  // state entries a thread requests
-constexpr int kRouteChunk = 8;  // float4 loads of W_r a thread issues before using them
-
-// The replacement of a one-token call by one whole warp on the block's copy of the cache state;
-// with publish (block 0) also the call's access record, counters and assignment records and the
-// layer's new state.
-__device__ __forceinline__ void route_replace(const Dev& d, int layer, const RouteSmem& r, uint64_t clock,
-                                              bool publish) {
-  const int lane = threadIdx.x & 31, E = d.E, S = d.S_active, k = d.k;
-  if (publish && lane == 0) d.info[2] = 0;
-  __syncwarp();
-  // one token: the k chosen experts are distinct, the accesses are them in rank order
-  lru_warp(d, layer, k, r.sel, r.slot_of, r.expert_of, r.last, r.uslot, clock, publish, r.umiss);
-  if (publish) {
-    if (lane < k) {  // one assignment per distinct expert: t = 0, j = u
-      d.pos_slot[lane] = r.uslot[lane];
-      d.asg[lane] = lane;
-      d.asg_off[lane] = lane;
-    }
-    if (lane == 0) d.asg_off[k] = k;
-    int32_t* g_slot_of = d.slot_of + (size_t)layer * E;
-    int32_t* g_expert_of = d.expert_of + (size_t)layer * d.S_alloc;
-    uint64_t* g_last = d.last_use + (size_t)layer * d.S_alloc;
-    for (int e = lane; e < E; e += 32) g_slot_of[e] = r.slot_of[e];
-    for (int q = lane; q < S; q += 32) {
-      g_expert_of[q] = r.expert_of[q];
-      g_last[q] = r.last[q];
-    }
-  }
-}
-
-// Every thread of the block calls it (block barriers inside), right after the kernel's wait for
-// the previous launch; rbase is the block's routing scratch (route_smem), epoch tags this call's
-// logits.  Out of line: its registers are allocated apart from the expert FFN's.
-__device__ __noinline__ void route_one_token(const Dev& d, int layer, const float* xs, uint64_t* xbar,
-                                             const float* __restrict__ wr, const float* __restrict__ bias, int wpe,
-                                             uint32_t epoch, unsigned char* rbase) {
-  const RouteSmem r = route_smem(rbase, d.E, d.S_alloc);
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int E = d.E, S = d.S_active, k = d.k, n4 = d.H / 4;
-  const int32_t* g_slot_of = d.slot_of + (size_t)layer * E;
-  const int32_t* g_expert_of = d.expert_of + (size_t)layer * d.S_alloc;
-  const uint64_t* g_last = d.last_use + (size_t)layer * d.S_alloc;
-  int pre_slot[kPreF], pre_exp[kPreF];
-  uint64_t pre_last[kPreF];
-#pragma unroll
-  for (int i = 0; i < kPreF; ++i) {
-    const int e = tid + i * kThreadsF;
-    pre_slot[i] = e < E ? g_slot_of[e] : -1;
-    pre_exp[i] = e < S ? g_expert_of[e] : -1;
-    pre_last[i] = e < S ? g_last[e] : 0;
-  }
-  const uint64_t clock0 = warp == 0 ? d.clock[layer] : 0;
-  const uint64_t pol = l2_evict_last();  // W_r is read again by the layer's next call
-  const float4* x4 = reinterpret_cast<const float4*>(xs);  // x, staged in shared memory
-  const int step = wpe * 32;
-  bool x_ready = false;
-  for (int e = blockIdx.x; e < E; e += gridDim.x) {  // block-uniform
-    const float4* w4 = reinterpret_cast<const float4*>(wr + (size_t)e * d.H);
-    float s = 0.f, c = 0.f;
-    if (tid < step)
-      for (int q0 = tid; q0 < n4; q0 += kRouteChunk * step) {
-        float4 a[kRouteChunk];
-#pragma unroll
-        for (int u = 0; u < kRouteChunk; ++u) {  // the chunk's W_r loads first
-          const int q = q0 + u * step;
-          if (q < n4) a[u] = ld_hint(w4 + q, pol);
-        }
-        if (!x_ready) {  // x's bulk copy (garbage on a timeout, never a hang)
-          x_ready = true;
-          if (!mbar_wait(xbar, 0, d.wait_ns)) atomicExch(d.err, 4u);
-        }
-#pragma unroll
-        for (int u = 0; u < kRouteChunk; ++u)
-          if (q0 + u * step < n4) {
-            const float4 b = x4[q0 + u * step];
-            dot2(s, c, a[u].x, b.x);
-            dot2(s, c, a[u].y, b.y);
-            dot2(s, c, a[u].z, b.z);
-            dot2(s, c, a[u].w, b.w);
-          }
-      }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float so = __shfl_xor_sync(0xffffffffu, s, off);
-      const float co = __shfl_xor_sync(0xffffffffu, c, off);
-      pair_add(s, c, so, co);
-    }
-    if (lane == 0 && warp < wpe) {
-      r.ps[warp] = s;
-      r.pc[warp] = c;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      float zs = r.ps[0], zc = r.pc[0];
-      for (int w = 1; w < wpe; ++w) pair_add(zs, zc, r.ps[w], r.pc[w]);
-      float z = __fadd_rn(zs, zc);
-      if (bias) z = __fadd_rn(z, bias[e]);
-      st_relaxed_u64(d.ztag + e, (unsigned long long)epoch << 32 | __float_as_uint(z));
-    }
-    __syncthreads();  // the partials are reused by the block's next expert
-  }
-#pragma unroll
-  for (int i = 0; i < kPreF; ++i) {  // the cache state (landed meanwhile) into shared memory
-    const int e = tid + i * kThreadsF;
-    if (e < E) r.slot_of[e] = pre_slot[i];
-    if (e < S) {
-      r.expert_of[e] = pre_exp[i];
-      r.last[e] = pre_last[i];
-    }
-  }
-  bool ok = true;
-  for (int e = tid; e < E; e += kThreadsF) {  // every block's logits, as each becomes visible
-    unsigned long long v = 0;
-    ok &= tagged_wait(d.ztag + e, epoch, d.wait_ns, v);
-    r.z[e] = __uint_as_float((uint32_t)v);
-  }
-  if (!ok) atomicExch(d.err, 5u);
-  rank_topk(r.z, E, k, r.sel, r.zsel);  // (block barrier first)
-  if (warp == 0) {
-    const bool pub = blockIdx.x == 0;
-    const float g = topk_softmax(r.zsel, k);
-    if (lane < k) r.g[lane] = g;
-    if (pub && lane < k) {
-      d.idx[lane] = r.sel[lane];
-      d.g[lane] = g;
-    }
-    const int sl = lane < k ? r.slot_of[r.sel[lane]] : 0;
-    if (__all_sync(0xffffffffu, sl >= 0)) {  // every access hits
-      if (lane < k) {
-        r.uslot[lane] = sl;
-        r.umiss[lane] = 0;
-      }
-      if (lane == 0) r.later[0] = pub ? 1 : 0;
-    } else {
-      if (lane == 0) r.later[0] = 0;
-      route_replace(d, layer, r, __shfl_sync(0xffffffffu, clock0, 0), pub);
-    }
-  }
-  __syncthreads();
-}
-
-// A float4 load the compiler keeps where it is written (it may not sink it past a call).
-__device__ __forceinline__ float4 ld_early(const float4* p) {
-  float4 v;
-  asm volatile("ld.global.nc.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "l"(p));
-  return v;
-}
-
-// ---- x split by the consumers, kG = kW / 4 threads (consecutive lanes) per group of x, each
-// thread one word of four values; kXR rounds of 512 words (the fused path takes H <= 4096).
-// The same pieces as quant_vals of the whole group: the group's largest magnitude m by shuffles,
-// each value scaled by 2^-e_g (e_g: m's exponent) and split by 127 / (m 2^-e_g), the piece sums
-// added over the kG threads; then the vector's exponent and rescale_group as in split_vectors.
-constexpr int kXR = 2;
-template <int QT>
-__device__ __forceinline__ void split_x_words(const float4 (&xv)[kXR], int n_words, XQ<QT>* dst, int* s_max,
-                                              int* s_exp) {
-  constexpr int kG = Vec<QT>::kW / 4;
-  int eg[kXR];
-#pragma unroll
-  for (int rr = 0; rr < kXR; ++rr) {
-    eg[rr] = kNoExp;
-    if (rr * kConsumers * 32 >= n_words) break;  // block-uniform
-    const int w = (int)threadIdx.x + rr * kConsumers * 32, gi = w / kG, part = w % kG;
-    const float4 v = xv[rr];
-    float m = fmaxf(fmaxf(fabsf(v.x), fabsf(v.y)), fmaxf(fabsf(v.z), fabsf(v.w)));
-#pragma unroll
-    for (int o = 1; o < kG; o <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-    eg[rr] = group_exponent(m);
-    const int ne = eg[rr] == kNoExp ? 0 : -eg[rr];
-    const float sa = pow2i(ne / 2), sb = pow2i(ne - ne / 2);
-    const float ms = m * sa * sb;  // exact: the largest value scaled by a power of two
-    const float inv = ms > 0x1p-100f ? 127.f / ms : 0.f;
-    const float vv[4] = {v.x * sa * sb, v.y * sa * sb, v.z * sa * sb, v.w * sa * sb};
-    uint32_t b1 = 0, b2 = 0, b3 = 0;
-    int s1 = 0, s2 = 0, s3 = 0;
-#pragma unroll
-    for (int jj = 0; jj < 4; ++jj) {
-      const float t = vv[jj] * inv;
-      const int a = __float2int_rn(t);
-      const float e = (t - (float)a) * 127.f;
-      const int b = __float2int_rn(e);
-      const int c = __float2int_rn((e - (float)b) * 127.f);
-      s1 += a;
-      s2 += b;
-      s3 += c;
-      b1 |= (uint32_t)(a & 0xFF) << (8 * jj);
-      b2 |= (uint32_t)(b & 0xFF) << (8 * jj);
-      b3 |= (uint32_t)(c & 0xFF) << (8 * jj);
-    }
-#pragma unroll
-    for (int o = 1; o < kG; o <<= 1) {
-      s1 += __shfl_xor_sync(0xffffffffu, s1, o);
-      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-      s3 += __shfl_xor_sync(0xffffffffu, s3, o);
-    }
-    if (w < n_words) {
-      dst[gi].p1[part] = b1;
-      dst[gi].p2[part] = b2;
-      dst[gi].p3[part] = b3;
-      if (part == 0) {
-        constexpr int off = QT == kQ8 ? 128 : 8;
-        dst[gi].k12 = off * (s1 * 127 + s2);
-        dst[gi].k3 = off * s3;
-        dst[gi].sf = inv > 0.f ? ms / 127.f / 16129.f : 0.f;
-      }
-    }
-    int wm = w < n_words ? eg[rr] : kNoExp;  // the warp's largest exponent: one shared atomic per warp
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) wm = max(wm, __shfl_xor_sync(0xffffffffu, wm, o));
-    if ((threadIdx.x & 31) == 0 && wm != kNoExp) atomicMax(s_max, wm);
-  }
-  named_bar_sync(1, kConsumers * 32);
-#pragma unroll
-  for (int rr = 0; rr < kXR; ++rr) {
-    const int w = (int)threadIdx.x + rr * kConsumers * 32;
-    if (w < n_words && w % kG == 0) rescale_group<QT>(dst[w / kG], eg[rr], vector_exponent(*s_max));
-  }
-  if (threadIdx.x == 0) *s_exp = vector_exponent(*s_max);
-  named_bar_sync(1, kConsumers * 32);
-}
-
 template <int QT, int VPL, int VPLD>
 __global__ void __launch_bounds__(kThreadsF, 1)
-    k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, const float* __restrict__ wr,
-               const float* __restrict__ bias, float* __restrict__ y, FusedCfg f) {
+    k_ffn_pipe(Dev d, int layer, const float* __restrict__ x, float* __restrict__ y, FusedCfg f) {
   constexpr int kW = Vec<QT>::kW;
   extern __shared__ __align__(128) unsigned char smem[];
   __shared__ uint8_t* s_gu[kMaxTopK];  // each expert's HBM slot: gate/up region, down region
@@ -727,7 +431,6 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   sm.full = reinterpret_cast<uint64_t*>(smem + f.off_bar);
   sm.empty = sm.full + kMaxStages;
   uint64_t* full_d = sm.empty + kMaxStages;  // [kMaxTopK] down buffers, one use each
-  uint64_t* xbar = full_d + kMaxTopK;         // x staged into the vq region (routed launches)
   unsigned char* dbuf = smem + f.off_dn;
   sm.red = reinterpret_cast<float*>(smem + f.off_red);
   sm.vq = smem + f.off_vq;
@@ -743,40 +446,15 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       mbar_init(&sm.empty[s], kConsumers);
     }
     for (int j = 0; j < k; ++j) mbar_init(&full_d[j], 1);
-    mbar_init(xbar, 1);
     mbar_fence_init();
     s_xmax = kNoExp;
   }
   if (threadIdx.x < kMaxTopK) s_hmax[threadIdx.x] = kNoExp;
-  __syncthreads();  // the barriers are initialised before any thread waits on one
-  pdl_wait();  // the previous launch (the router, or the previous call) is complete and visible
-  // consumer thread t: words t, t + 512 of x (four values each), requested while the block sets up
-  const int n_xw = d.H / 4;
-  float4 xv[kXR];
-#pragma unroll
-  for (int rr = 0; rr < kXR; ++rr) {  // (volatile: issued here, before the expert weights' flood)
-    const int w = (int)threadIdx.x + rr * kConsumers * 32;
-    xv[rr] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (!f.route && warp < kConsumers && w < n_xw) xv[rr] = ld_early(reinterpret_cast<const float4*>(x) + w);
-  }
-  if (f.route && threadIdx.x == 0) {  // routed: x (device memory) into the vq region, one bulk copy
-    mbar_arrive_tx(xbar, (uint32_t)d.H * 4u);
-    bulk_g2s(sm.vq, x, (uint32_t)d.H * 4u, xbar);
-  }
-  if (f.route) {  // the token's routing and slot replacement, in this launch
-    const RouteSmem r = route_smem(smem + f.off_route, d.E, d.S_alloc);
-    const uint32_t epoch = (uint32_t)d.work[1] + 1;  // this call's tag: the previous call's + 1
-    route_one_token(d, layer, reinterpret_cast<const float*>(sm.vq), xbar, wr, bias, f.wpe, epoch, smem + f.off_route);
-    if (threadIdx.x < k) {
-      const int j = threadIdx.x;
-      uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + r.uslot[j]) * d.lay.stride;
-      s_gu[j] = slot;
-      s_dn[j] = slot + d.lay.d_off;
-      s_hgu[j] = d.pack + ((size_t)layer * d.E + r.sel[j]) * d.lay.stride;
-      s_g[j] = r.g[j];
-      s_miss[j] = r.umiss[j];
-    }
-  } else if (threadIdx.x < k) {  // one token, routed by the router: access u = rank j
+  pdl_wait();  // the router's outputs (and the caller's x) are complete and visible
+  float xv[kW];  // consumer thread i < n_vec: group i of x, requested while the block sets up
+  const bool x_mine = warp < kConsumers && (int)threadIdx.x < cg.n_vec;
+  if (x_mine) load_group<QT>(x + (size_t)threadIdx.x * kW, xv);
+  if (threadIdx.x < k) {  // one token: access u = rank j
     uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
     s_gu[threadIdx.x] = slot;
     s_dn[threadIdx.x] = slot + d.lay.d_off;
@@ -786,25 +464,24 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     s_miss[threadIdx.x] = d.umiss[threadIdx.x];
   }
   __syncthreads();
-  if (warp == 0) {
-    // list position p = blockIdx.x + t * gridDim.x (lane t); the list holds the resident experts'
-    // items, then the missed experts' (ranks in order within each); item id = rank * (I / R) + row
-    // block.  Position q of the expert list: the q-th resident rank, or the (q - n_res)-th missed one.
+  if (threadIdx.x == 0) {
+    // list position p = blockIdx.x + t * gridDim.x; the list holds the resident experts' items,
+    // then the missed experts' (ranks in order within each); item id = rank * (I / R) + row block
     const int nrb = d.I / cg.R;
-    const unsigned kmask = (1u << k) - 1u;
-    const unsigned res = __ballot_sync(0xffffffffu, lane < k && !s_miss[lane]);
-    const int n_res_e = __popc(res);
-    for (int t = lane; t < mine_g; t += 32) {
-      const int p = (int)blockIdx.x + t * (int)gridDim.x, q = p / nrb;
-      unsigned m = q < n_res_e ? res : (~res & kmask);
-      for (int c = q < n_res_e ? q : q - n_res_e; c > 0; --c) m &= m - 1u;  // drop the c lowest ranks
-      s_gord[t] = (__ffs(m) - 1) * nrb + p % nrb;
+    int* ord = s_ord;
+    int n_res_e = 0;
+    for (int j = 0; j < k; ++j)
+      if (!s_miss[j]) ord[n_res_e++] = j;
+    for (int j = 0, n = n_res_e; j < k; ++j)
+      if (s_miss[j]) ord[n++] = j;
+    int nres = 0;
+    for (int t = 0; t < mine_g; ++t) {
+      const int p = (int)blockIdx.x + t * (int)gridDim.x;
+      s_gord[t] = ord[p / nrb] * nrb + p % nrb;
+      nres += p < n_res_e * nrb;
     }
-    if (lane == 0) {
-      const int lim = n_res_e * nrb - (int)blockIdx.x;  // items t with p < n_res_e * nrb
-      s_nres = lim <= 0 ? 0 : min(mine_g, (lim + (int)gridDim.x - 1) / (int)gridDim.x);
-      s_nb = n_res_e < k ? 2 : 0;  // ring B only when the call has a missed expert (NS >= 4)
-    }
+    s_nres = nres;
+    s_nb = n_res_e < k ? 2 : 0;  // ring B only when the call has a missed expert (NS >= 4)
   }
   __syncthreads();
 
@@ -858,10 +535,6 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     // ---- link warp: the missed experts' items through ring B (both stages in flight at once),
     // then all their down records at once (after the items: the grid barrier and the h split
     // overlap that transfer)
-    if (f.route && blockIdx.x == 0) {  // every access hit: the replacement's bookkeeping, here
-      const RouteSmem r = route_smem(smem + f.off_route, d.E, d.S_alloc);
-      if (r.later[0]) route_replace(d, layer, r, d.clock[layer], true);
-    }
     bool ok = true;
     const int R = cg.R, nrb = d.I / R, n_li = mine_g - nres;
     const uint32_t bytes = cg.stage_bytes, rs = d.lay.rs_gu;
@@ -930,17 +603,18 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       const int nv = (d.lay.qrow_gu / 16) / cs;
       const int v0 = col * nv;
       const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-      if (f.route) {  // x from its staged copy, read by every consumer before the split overwrites it
-        if (!mbar_wait(xbar, 0, d.wait_ns) && lane == 0) atomicExch(d.err, 4u);  // (garbage, no hang)
-#pragma unroll
-        for (int rr = 0; rr < kXR; ++rr) {
-          const int w = (int)threadIdx.x + rr * kConsumers * 32;
-          if (w < n_xw) xv[rr] = reinterpret_cast<const float4*>(sm.vq)[w];
+      {  // x split into int8 pieces, scaled by the power of two of its largest magnitude
+        XQ<QT>* dst = reinterpret_cast<XQ<QT>*>(sm.vq);
+        const int eg = x_mine ? group_exponent(group_absmax<QT>(xv)) : kNoExp;
+        if (x_mine) {
+          dst[threadIdx.x] = quant_vals<QT>(xv, eg == kNoExp ? 0 : -eg);
+          atomicMax(&s_xmax, eg);
         }
         named_bar_sync(1, kConsumers * 32);
+        if (x_mine) rescale_group<QT>(dst[threadIdx.x], eg, vector_exponent(s_xmax));
+        if (threadIdx.x == 0) s_xexp = vector_exponent(s_xmax);
+        named_bar_sync(1, kConsumers * 32);
       }
-      // x split into int8 pieces, scaled by the power of two of its largest magnitude
-      split_x_words<QT>(xv, n_xw, reinterpret_cast<XQ<QT>*>(sm.vq), &s_xmax, &s_xexp);
       XQ<QT> xr[VPL];
 #pragma unroll
       for (int i = 0; i < VPL; ++i) {
@@ -1054,8 +728,6 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     }
   }
   __syncthreads();
-  // every block has read this call's epoch (block 0 passed the grid-wide wait for all of them)
-  if (f.route && blockIdx.x == 0 && threadIdx.x == 0) d.work[1] += 1;  // the next call's epoch
 }
 
 int vpl_for(int nvec) {
@@ -1162,10 +834,8 @@ cudaError_t down_pipe_q(const Dev& d, int layer, float* y, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-FusedCfg fused_cfg(const Dev& d, bool route) {
+FusedCfg fused_cfg(const Dev& d) {
   FusedCfg f;
-  f.route = route ? 1 : 0;
-  f.wpe = route ? router_warps_per_expert(d.E, d.H) : 0;
   f.g = gateup_cfg(d);
   f.rpc = (d.H + sm_count() - 1) / sm_count();
   f.dn_bytes = (uint32_t)f.rpc * d.lay.rs_d;
@@ -1174,34 +844,28 @@ FusedCfg fused_cfg(const Dev& d, bool route) {
   f.stage_bytes = f.g.stage_bytes;
   f.red_floats = f.g.max_mine * kConsumers + d.k * f.rpc;
   f.vq_bytes = f.g.vq_bytes > hv_bytes ? f.g.vq_bytes : hv_bytes;
-  if (route && f.vq_bytes < (uint32_t)d.H * 4u) f.vq_bytes = (uint32_t)d.H * 4u;  // x is staged there first
-  const size_t rbytes = route ? route_bytes(d.E, d.S_alloc) : 0;
   const size_t fixed = (size_t)d.k * f.dn_bytes + kFusedBars * sizeof(uint64_t) +
-                       (size_t)f.red_floats * sizeof(float) + f.vq_bytes + 64 + rbytes;  // (+ alignment)
+                       (size_t)f.red_floats * sizeof(float) + f.vq_bytes;
   const size_t budget = kFusedSmem - 1024;  // - the kernel's static shared memory
   const size_t ns = fixed < budget ? (budget - fixed) / f.stage_bytes : 0;
   f.NS = (int)(ns > (size_t)kMaxStages ? kMaxStages : ns);
-  // every region starts on a 16-byte boundary (bulk copies and 16-byte accesses into stages, the
-  // down buffers and vq)
-  auto a16 = [](size_t v) { return (v + 15) & ~(size_t)15; };
-  f.off_dn = a16((size_t)f.NS * f.stage_bytes);
-  f.off_bar = a16(f.off_dn + (size_t)d.k * f.dn_bytes);
-  f.off_red = a16(f.off_bar + kFusedBars * sizeof(uint64_t));
-  f.off_vq = a16(f.off_red + (size_t)f.red_floats * sizeof(float));
-  f.off_route = a16(f.off_vq + f.vq_bytes);
-  f.total = f.off_route + rbytes;
+  f.off_dn = (size_t)f.NS * f.stage_bytes;
+  f.off_bar = f.off_dn + (size_t)d.k * f.dn_bytes;
+  f.off_red = f.off_bar + kFusedBars * sizeof(uint64_t);
+  f.off_vq = f.off_red + (((size_t)f.red_floats * sizeof(float) + 15) & ~(size_t)15);
+  f.total = f.off_vq + f.vq_bytes;
   return f;
 }
 
 size_t fused_smem(const FusedCfg& f) { return f.total; }
 
-// One block per SM.  The launch is programmatic (it may begin while the previous kernel of the
-// stream finishes: the kernel's prologue touches only shared memory and it waits for that kernel
-// before reading anything else); where the driver refuses that, a cooperative launch.  Blocks
-// wait for each other only through bounded waits.
+// One block per SM.  The launch is programmatic (it may begin while the router finishes: the
+// kernel's prologue touches only shared memory and it waits for the router before reading
+// anything else); where the driver refuses that, a cooperative launch.  Blocks wait for each
+// other only through bounded waits.
 template <class Kern>
-cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x,
-                       const float* wr, const float* bias, float* y, const FusedCfg& f) {
+cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int layer, const float* x, float* y,
+                       const FusedCfg& f) {
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -1216,24 +880,23 @@ cudaError_t launch_ffn(Kern kern, size_t smem, cudaStream_t s, const Dev& d, int
   if (pdl_ok) {
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
-    e = cudaLaunchKernelEx(&cfg, kern, d, layer, x, wr, bias, y, f);
+    e = cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
     if (e == cudaSuccess) return e;
     cudaGetLastError();
     pdl_ok = false;
   }
   attr[0].id = cudaLaunchAttributeCooperative;  // every block resident: they wait for each other
   attr[0].val.cooperative = 1;
-  return cudaLaunchKernelEx(&cfg, kern, d, layer, x, wr, bias, y, f);
+  return cudaLaunchKernelEx(&cfg, kern, d, layer, x, y, f);
 }
 
 template <int QT>
-cudaError_t ffn_pipe_q(const Dev& d, int layer, const float* x, const float* wr, const float* bias, float* y,
-                       cudaStream_t s) {
-  const FusedCfg f = fused_cfg(d, wr != nullptr);
+cudaError_t ffn_pipe_q(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
+  const FusedCfg f = fused_cfg(d);
   const size_t smem = fused_smem(f);
   const int vx = vpl_for((d.lay.qrow_gu / 16) / f.g.cs), vh = vpl_for(d.lay.qrow_d / 16);
 #define MF_FF(A, B) \
-  if (vx == A && vh == B) return launch_ffn(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, wr, bias, y, f);
+  if (vx == A && vh == B) return launch_ffn(k_ffn_pipe<QT, A, B>, smem, s, d, layer, x, y, f);
   MF_FF(1, 1) MF_FF(1, 2) MF_FF(2, 1) MF_FF(2, 2)
   if constexpr (QT == kQ8) {  // Q4_0 takes at most two vectors per lane (decode_pipe_ok)
     MF_FF(1, 3) MF_FF(2, 3) MF_FF(3, 1) MF_FF(3, 2) MF_FF(3, 3) MF_FF(4, 1) MF_FF(4, 2) MF_FF(4, 3)
@@ -1268,24 +931,12 @@ cudaError_t launch_down_single_pipe(const Dev& d, int layer, float* y, cudaStrea
 size_t decode_smem_bytes(const Dev& d, int which) { return smem_bytes(which == 0 ? gateup_cfg(d) : down_cfg(d)); }
 
 bool ffn_fused_ok(const Dev& d) {
-  const FusedCfg f = fused_cfg(d, false);
-  return decode_pipe_ok(d) && f.NS >= 4 && f.g.max_mine <= kMaxItemsF && d.H / 4 <= kXR * kConsumers * 32 &&
-         f.stage_bytes % 16 == 0 && f.dn_bytes % 16 == 0;
-}
-
-bool ffn_routed_ok(const Dev& d) {
-  return ffn_fused_ok(d) && fused_cfg(d, true).NS >= 4 && d.E <= kMaxExperts;
+  const FusedCfg f = fused_cfg(d);
+  return decode_pipe_ok(d) && f.NS >= 4 && f.g.max_mine <= kMaxItemsF;
 }
 
 cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s) {
-  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, nullptr, nullptr, y, s)
-                            : ffn_pipe_q<kQ4>(d, layer, x, nullptr, nullptr, y, s);
-}
-
-cudaError_t launch_ffn_routed(const Dev& d, int layer, const float* x, const float* wr, const float* bias, float* y,
-                              cudaStream_t s) {
-  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, wr, bias, y, s)
-                            : ffn_pipe_q<kQ4>(d, layer, x, wr, bias, y, s);
+  return d.qtype == MF_Q8_0 ? ffn_pipe_q<kQ8>(d, layer, x, y, s) : ffn_pipe_q<kQ4>(d, layer, x, y, s);
 }
 
 }  // namespace mf

@@ -59,8 +59,6 @@ struct Dev {
   uint8_t* tr_hit;     // [L][E]
   // per-call scratch
   float2* zpart;       // router, T >= kTiledMinT: compensated logit pairs [K split][T][E]
-  unsigned long long* ztag;  // [E]     logits of a one-token call routed inside the fused kernel,
-                             //           each with the call's epoch in its upper 32 bits
   int32_t* idx;        // [T_max][k]
   float* g;            // [T_max][k]
   int32_t* uniq;       // [E]           distinct experts in access order
@@ -79,8 +77,7 @@ struct Dev {
   uint8_t* xt;         // x tiles:  t * (H / 32) + kk
   uint8_t* ht;         // h tiles:  t * (I / 32) + kk
   uint8_t* stage;      // [S_alloc] payloads: a wave's misses staged while the previous wave computes (T_max > 1)
-  unsigned long long* work;  // [16]     arrival counter of the fused one-token FFN kernel (word 0),
-                             //           epoch of the latest routed call (word 1)
+  unsigned long long* work;  // [16]     arrival counter of the fused one-token FFN kernel (word 0)
   unsigned* err;       // [1]           nonzero after a bounded wait gave up (see MF_E_TIMEOUT)
   uint64_t wait_ns;    // time limit of every bounded device wait (mf_wait_limit)
   int hold;            // test hold (mf_test_hold): the fused FFN's producer issues no copies
@@ -153,29 +150,6 @@ __device__ __forceinline__ bool counter_wait(const unsigned long long* cnt, unsi
       if (gtimer_ns() - t0 > limit_ns) return false;
       __nanosleep(32);
     }
-  }
-  return false;
-}
-// Relaxed (gpu scope) 64-bit accesses: single-copy atomic, no ordering, no fence.
-__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long* p) {
-  unsigned long long v;
-  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ void st_relaxed_u64(unsigned long long* p, unsigned long long v) {
-  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
-}
-// Bounded wait until the word at p carries `tag` in its upper 32 bits (the word is its own flag);
-// the word in v.  false once `limit_ns` nanoseconds have passed.
-__device__ __forceinline__ bool tagged_wait(const unsigned long long* p, uint32_t tag, uint64_t limit_ns,
-                                            unsigned long long& v) {
-  v = ld_relaxed_u64(p);
-  if ((uint32_t)(v >> 32) == tag) return true;
-  const uint64_t t0 = gtimer_ns();
-  for (uint32_t i = 0; i < kWaitPolls; ++i) {
-    v = ld_relaxed_u64(p);
-    if ((uint32_t)(v >> 32) == tag) return true;
-    if (gtimer_ns() - t0 > limit_ns) return false;
   }
   return false;
 }
@@ -270,7 +244,6 @@ struct mf_ctx {
   uint64_t overhead_bytes;
   bool decode_pipe;  // batch-1 calls use the pipelined decode kernels
   bool ffn_fused;    // ... fused into one cooperative launch
-  bool ffn_routed;   // ... with the token's routing inside that launch (device x, pinned pack)
   int prefill_min_t;  // calls with T >= this use the tensor-core grouped GEMMs (0 = never)
   uint8_t* gemm_scratch;  // x and h tiles of the tensor-core path (allocated when first enabled)
   bool tmaps_ok;
@@ -312,13 +285,6 @@ bool decode_pipe_ok(const Dev& d);
 // both projections of one token in one cooperative launch (d.work holds its arrival counter)
 bool ffn_fused_ok(const Dev& d);
 cudaError_t launch_ffn_single(const Dev& d, int layer, const float* x, float* y, cudaStream_t s);
-// one-token call, routed inside the fused kernel (router, slot replacement and expert FFN in one
-// launch), with the one-token router's arithmetic order
-int router_cluster_size(int H);
-int router_warps_per_expert(int E, int H);
-bool ffn_routed_ok(const Dev& d);
-cudaError_t launch_ffn_routed(const Dev& d, int layer, const float* x, const float* wr, const float* bias, float* y,
-                              cudaStream_t s);
 // many tokens per expert: tcgen05 grouped GEMMs (gate/up + SwiGLU, down) per wave
 constexpr int kPrefillMinTokens = 256;
 bool prefill_shape_ok(int hidden, int inter);

@@ -16,13 +16,10 @@ namespace mf {
 constexpr int kMissBit = 1 << 30;  // in s_uslot until the record is written
 
 // The record of every access (uniq, uslot, umiss, trace) and the counters, from s_uslot (slot,
-// with kMissBit for a miss); clears the bit and, where s_umiss is given, keeps each access's miss
-// flag there.  All 32 lanes of one warp call it; lane 0's clock and eviction count are the ones
-// stored.  Without publish nothing goes to global memory (a block that replays the replacement
-// for its own use).
+// with kMissBit for a miss); clears the bit.  All 32 lanes of one warp call it; lane 0's clock
+// and eviction count are the ones stored.
 __device__ __forceinline__ void lru_records(const Dev& d, int layer, int U, const int* s_uniq, int* s_uslot,
-                                            uint64_t clock, uint64_t evictions, bool publish = true,
-                                            int* s_umiss = nullptr) {
+                                            uint64_t clock, uint64_t evictions) {
   const int lane = threadIdx.x & 31, E = d.E, S = d.S_active;
   unsigned misses = 0;
   for (int u0 = 0; u0 < U; u0 += 32) {  // warp-uniform: every lane takes part in the ballot
@@ -32,10 +29,9 @@ __device__ __forceinline__ void lru_records(const Dev& d, int layer, int U, cons
     const bool miss = valid && (s & kMissBit);
     s &= ~kMissBit;
     misses += __popc(__ballot_sync(0xffffffffu, miss));
-    if (valid) s_uslot[u] = s;
-    if (valid && s_umiss) s_umiss[u] = miss ? 1 : 0;
-    if (valid && publish) {
+    if (valid) {
       const int e = s_uniq[u];
+      s_uslot[u] = s;
       d.uniq[u] = e;
       d.uslot[u] = s;
       d.umiss[u] = miss ? 1 : 0;
@@ -45,7 +41,7 @@ __device__ __forceinline__ void lru_records(const Dev& d, int layer, int U, cons
     }
   }
   __syncwarp();
-  if (lane == 0 && publish) {
+  if (lane == 0) {
     const uint64_t hits = (uint64_t)U - misses;
     d.clock[layer] = clock;
     unsigned long long* st = reinterpret_cast<unsigned long long*>(d.stats + (size_t)layer * 5);
@@ -64,11 +60,9 @@ __device__ __forceinline__ void lru_records(const Dev& d, int layer, int U, cons
 // Writes the call's access record (uniq, uslot, umiss, trace), per-wave miss lists and counts,
 // the counters and the clock.  All 32 lanes must call it.  The accesses are decided one after
 // the other (lane 0 updates the state; the warp searches free and least-recently-used slots);
-// the record of every access is then written by the whole warp at once.  publish and s_umiss as
-// for lru_records.
+// the record of every access is then written by the whole warp at once.
 __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const int* s_uniq, int* s_slot_of,
-                                         int* s_expert_of, uint64_t* s_last, int* s_uslot, uint64_t clock,
-                                         bool publish = true, int* s_umiss = nullptr) {
+                                         int* s_expert_of, uint64_t* s_last, int* s_uslot, uint64_t clock) {
   const int lane = threadIdx.x & 31, S = d.S_active;  // the clock is kept by lane 0
   uint64_t evictions = 0;
   int wave = 0, wpos = 0, wave_miss = 0;  // wave of access u, u's position in it, misses so far in it
@@ -89,7 +83,7 @@ __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const i
       }
     }
     clock += (uint64_t)U;
-    if (lane == 0 && publish)
+    if (lane == 0)
       for (int w = 0; w * S < U; ++w) d.info[2 + w] = 0;
     __syncwarp();
   }
@@ -129,7 +123,7 @@ __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const i
       if (lane == 0) {
         s_expert_of[s] = e;
         s_slot_of[e] = s;
-        if (publish) d.miss_list[wave * S + wave_miss] = u;
+        d.miss_list[wave * S + wave_miss] = u;
       }
       ++wave_miss;
     }
@@ -138,14 +132,14 @@ __device__ __forceinline__ void lru_warp(const Dev& d, int layer, int U, const i
       s_uslot[u] = hit ? s : (s | kMissBit);
     }
     if (++wpos == S || u == U - 1) {  // end of a wave: its miss count
-      if (lane == 0 && publish) d.info[2 + wave] = wave_miss;
+      if (lane == 0) d.info[2 + wave] = wave_miss;
       ++wave;
       wpos = 0;
       wave_miss = 0;
     }
     __syncwarp();  // lane 0's shared-memory updates are seen by the whole warp at the next access
   }
-  lru_records(d, layer, U, s_uniq, s_uslot, clock, evictions, publish, s_umiss);
+  lru_records(d, layer, U, s_uniq, s_uslot, clock, evictions);
 }
 
 

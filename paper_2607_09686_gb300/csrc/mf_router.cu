@@ -1,7 +1,12 @@
-// Router: logits z = W_r x (+ bias), top-k by (z desc, id asc), softmax over the chosen
-// (Background section of the paper; the compensated arithmetic, the ranking and the softmax are
-// in mf_route.cuh).  One-token calls whose expert FFN runs fused take their routing inside that
-// kernel instead (mf_decode.cu); this kernel serves the other one-token calls.
+// Router: logits z = W_r x (+ bias), top-k by (z desc, id asc), softmax over the chosen.
+//
+// MoE routing selects a subset of experts per token (Background section of the paper).
+// Logits are computed with a compensated dot product (Ogita, Rump & Oishi, "Accurate sum and
+// dot product", SIAM J. Sci. Comput. 2005, algorithm Dot2): every product is split exactly
+// into value + error with an FMA, the running sum is kept as an unevaluated pair, and the pair
+// is rounded to fp32 once.  The result is the fp32 rounding of the exact dot product except
+// where the exact value lies within ~n*2^-48 relative of a rounding boundary, so selection does
+// not depend on the summation order.
 //
 // One thread-block cluster of 16 blocks per token (8 where the GPU does not schedule clusters of
 // 16): block r computes the logits of experts [r*ceil(E/nc), (r+1)*ceil(E/nc)), with
@@ -19,7 +24,6 @@
 #include <cooperative_groups.h>
 
 #include "mf_lru.cuh"
-#include "mf_route.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -30,6 +34,33 @@ constexpr int kThreadsR = 512;
 constexpr int kWarpsR = kThreadsR / 32;
 constexpr int kChunk = 8;  // float4 loads of W (and of x) a lane issues before using them
 constexpr int kPre = kMaxExperts / kThreadsR;  // prefetched cache-state entries per thread
+
+struct F2 {
+  float hi, lo;
+};
+
+__device__ __forceinline__ F2 two_sum(float a, float b) {
+  float s = __fadd_rn(a, b);
+  float bb = __fsub_rn(s, a);
+  float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return {s, e};
+}
+
+// (s, c) += a * b, error-free product split plus compensated running sum
+__device__ __forceinline__ void dot2(float& s, float& c, float a, float b) {
+  float p = __fmul_rn(a, b);
+  float pe = __fmaf_rn(a, b, -p);
+  F2 t = two_sum(s, p);
+  s = t.hi;
+  c = __fadd_rn(c, __fadd_rn(t.lo, pe));
+}
+
+// (s, c) += (s2, c2) for compensated pairs
+__device__ __forceinline__ void pair_add(float& s, float& c, float s2, float c2) {
+  const F2 t = two_sum(s, s2);
+  s = t.hi;
+  c = __fadd_rn(__fadd_rn(c, c2), t.lo);
+}
 
 // The first chunk of logit_part's W loads, issued before x is in shared memory.
 __device__ __forceinline__ void w_preload(const float* __restrict__ w, int n4, int first, int step, float4* a) {
@@ -182,12 +213,41 @@ __global__ void __launch_bounds__(kThreadsR)
   if (rank != 0) return;
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 
-  rank_topk(s_z, E, k, s_sel, s_zsel);
-  if (warp == 0) {
-    const float g = topk_softmax(s_zsel, k);
+  // rank by counting: position of expert e = experts with a larger logit, or equal and lower id
+  // (s_sel starts as 0..k-1: a valid choice even where the logits are not ordered, e.g. NaN).
+  // tpe consecutive lanes share an expert, each counting over every tpe-th other expert.
+  if (tid < k) s_sel[tid] = tid;
+  __syncthreads();
+  {
+    int tpe = 1;
+    while (tpe < 32 && tpe * 2 * E <= kThreadsR) tpe *= 2;
+    const int per_pass = kThreadsR / tpe, part = tid % tpe;
+    for (int e0 = 0; e0 < E; e0 += per_pass) {  // block-uniform
+      const int e = e0 + tid / tpe;
+      const bool valid = e < E;
+      const float z = valid ? s_z[e] : 0.f;
+      int r = 0;
+      if (valid)
+        for (int e2 = part; e2 < E; e2 += tpe) {
+          const float z2 = s_z[e2];
+          r += (z2 > z) || (z2 == z && e2 < e);
+        }
+      for (int off = tpe >> 1; off > 0; off >>= 1) r += __shfl_xor_sync(0xffffffffu, r, off);
+      if (valid && part == 0 && r < k) {
+        s_sel[r] = e;
+        s_zsel[r] = z;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {  // softmax over the chosen: lane j < k holds exp(z_j - z_0); fixed shuffle-tree sum
+    const float ex = lane < k ? expf(s_zsel[lane] - s_zsel[0]) : 0.f;
+    float den = ex;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) den += __shfl_xor_sync(0xffffffffu, den, off);
     if (lane < k) {
       d.idx[(size_t)t * k + lane] = s_sel[lane];
-      d.g[(size_t)t * k + lane] = g;
+      d.g[(size_t)t * k + lane] = ex / den;
     }
   }
   if (!resolve) return;
@@ -431,41 +491,6 @@ size_t router_part_pairs(int T_max, int E, int H) {
   return most;
 }
 
-// The one-token router's cluster size: 16 where the GPU can hold such a cluster (asked once, by
-// the first caller), else the portable 8.
-int router_cluster_size(int H) {
-  static int nc = 0;
-  if (nc == 0) {
-    nc = 8;
-    const size_t smem = (size_t)H * sizeof(float);
-    if (cudaFuncSetAttribute(k_router, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) == cudaSuccess &&
-        cudaFuncSetAttribute(k_router, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
-      cudaLaunchConfig_t cfg = {};
-      cfg.blockDim = dim3(kThreadsR);
-      cfg.dynamicSmemBytes = smem;
-      cfg.gridDim = dim3(16, 1);
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = 16;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      int clusters = 0;
-      if (cudaOccupancyMaxActiveClusters(&clusters, k_router, &cfg) == cudaSuccess && clusters >= 1) nc = 16;
-    }
-    cudaGetLastError();
-  }
-  return nc;
-}
-
-// Warps of one router block that share an expert's dot product (k_router: the block's epc
-// experts over its 16 warps).
-int router_warps_per_expert(int E, int H) {
-  const int epc = (E + router_cluster_size(H) - 1) / router_cluster_size(H);
-  return epc >= kWarpsR ? 1 : kWarpsR / epc;
-}
-
 cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const float* bias, int T, int layer,
                           cudaStream_t s, float* x_copy) {
   if (T >= kTiledMinT) return launch_router_tiled(d, x, wr, bias, T, s);
@@ -482,7 +507,18 @@ cudaError_t launch_router(const Dev& d, const float* x, const float* wr, const f
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  const int nc = router_cluster_size(d.H);
+  // cluster size: 16 where the GPU can hold such a cluster (asked once), else the portable 8
+  static int nc = 0;
+  if (nc == 0) {
+    nc = 8;
+    if (cudaFuncSetAttribute(k_router, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+      cfg.gridDim = dim3(16, 1);
+      attr[0].val.clusterDim.x = 16;
+      int clusters = 0;
+      if (cudaOccupancyMaxActiveClusters(&clusters, k_router, &cfg) == cudaSuccess && clusters >= 1) nc = 16;
+    }
+    cudaGetLastError();
+  }
   cfg.gridDim = dim3(nc, T);
   attr[0].val.clusterDim.x = nc;
   // programmatic: the launch may begin while the previous kernel of the stream finishes (the

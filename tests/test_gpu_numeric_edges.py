@@ -1,7 +1,6 @@
 """Numeric edge cases of the expert FFN against the CPU oracle, on every kernel path: the fused
-one-token launch (routed inside, or after the router kernel), the two pipelined one-token
-kernels, the one-warp-per-row kernels, the batched GEMV path (T = 4) and the tensor-core grouped
-GEMMs (T = 256).
+one-token launch, the two pipelined one-token kernels, the one-warp-per-row kernels, the batched
+GEMV path (T = 4) and the tensor-core grouped GEMMs (T = 256).
 
 The oracle computes in fp64 and rounds once (section "Native Serving Path": the expert FFN on the
 dequantised GGUF blocks); the GPU must meet the same tolerance on inputs far from the synthetic
@@ -87,7 +86,7 @@ CASES = {
     "scales_zero_subnormal": (edit_scales, lambda x: x, (Q8, Q4)),
     "h_zero_rows": (edit_gate_rows_zero, lambda x: x, (Q8, Q4)),
 }
-PATHS = ("fused", "fused_router", "pipelined", "simple", "batched", "prefill")
+PATHS = ("fused", "pipelined", "simple", "batched", "prefill")
 
 
 def tiny_scale(qtype, path):
@@ -106,8 +105,6 @@ def _run(path, case, qtype, monkeypatch):
     edit_fn, xform, qtypes = CASES[case]
     if qtype not in qtypes:
         pytest.skip("case applies to the other block format")
-    if path == "fused_router":
-        monkeypatch.setenv("MF_DECODE_ROUTER", "1")
     if path == "pipelined":
         monkeypatch.setenv("MF_DECODE_UNFUSED", "1")
     if path == "simple":
