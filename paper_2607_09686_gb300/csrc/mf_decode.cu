@@ -451,9 +451,14 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   }
   if (threadIdx.x < kMaxTopK) s_hmax[threadIdx.x] = kNoExp;
   pdl_wait();  // the router's outputs (and the caller's x) are complete and visible
-  float xv[kW];  // consumer thread i < n_vec: group i of x, requested while the block sets up
-  const bool x_mine = warp < kConsumers && (int)threadIdx.x < cg.n_vec;
-  if (x_mine) load_group<QT>(x + (size_t)threadIdx.x * kW, xv);
+  // x split by kG = kW / 4 threads per group (consecutive lanes), each one word of four values,
+  // where x has at most 512 words (H <= 2048); consumer thread t's word is requested while the
+  // block sets up.  Larger x: one group per thread (split_vectors).
+  constexpr int kG = kW / 4;
+  const bool x_words = cg.n_vec * kG <= kConsumers * 32;
+  const bool x_mine = x_words && warp < kConsumers && (int)threadIdx.x < cg.n_vec * kG;
+  float4 xv = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (x_mine) xv = __ldg(reinterpret_cast<const float4*>(x) + threadIdx.x);
   if (threadIdx.x < k) {  // one token: access u = rank j
     uint8_t* slot = d.pool + ((size_t)layer * d.S_alloc + d.uslot[threadIdx.x]) * d.lay.stride;
     s_gu[threadIdx.x] = slot;
@@ -603,17 +608,61 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       const int nv = (d.lay.qrow_gu / 16) / cs;
       const int v0 = col * nv;
       const XQ<QT>* xq = reinterpret_cast<const XQ<QT>*>(sm.vq);
-      {  // x split into int8 pieces, scaled by the power of two of its largest magnitude
+      if (x_words) {  // x split into int8 pieces, scaled by the power of two of its largest magnitude:
+                      // the same pieces as quant_vals of the whole group (the group's largest
+                      // magnitude m by shuffles, each value scaled by 2^-e_g and split by
+                      // 127 / (m 2^-e_g), the piece sums added over the kG threads), then the
+                      // vector's exponent and rescale_group as in split_vectors
         XQ<QT>* dst = reinterpret_cast<XQ<QT>*>(sm.vq);
-        const int eg = x_mine ? group_exponent(group_absmax<QT>(xv)) : kNoExp;
+        const int gi = threadIdx.x / kG, part = threadIdx.x % kG;
+        float m = fmaxf(fmaxf(fabsf(xv.x), fabsf(xv.y)), fmaxf(fabsf(xv.z), fabsf(xv.w)));
+#pragma unroll
+        for (int o = 1; o < kG; o <<= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        const int eg = group_exponent(m), ne = eg == kNoExp ? 0 : -eg;
+        const float sa = pow2i(ne / 2), sb = pow2i(ne - ne / 2);
+        const float ms = m * sa * sb;  // exact: the largest value scaled by a power of two
+        const float inv = ms > 0x1p-100f ? 127.f / ms : 0.f;
+        const float vv[4] = {xv.x * sa * sb, xv.y * sa * sb, xv.z * sa * sb, xv.w * sa * sb};
+        uint32_t b1 = 0, b2 = 0, b3 = 0;
+        int s1 = 0, s2 = 0, s3 = 0;
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) {
+          const float t = vv[jj] * inv;
+          const int a = __float2int_rn(t);
+          const float e = (t - (float)a) * 127.f;
+          const int b = __float2int_rn(e);
+          const int c = __float2int_rn((e - (float)b) * 127.f);
+          s1 += a;
+          s2 += b;
+          s3 += c;
+          b1 |= (uint32_t)(a & 0xFF) << (8 * jj);
+          b2 |= (uint32_t)(b & 0xFF) << (8 * jj);
+          b3 |= (uint32_t)(c & 0xFF) << (8 * jj);
+        }
+#pragma unroll
+        for (int o = 1; o < kG; o <<= 1) {
+          s1 += __shfl_xor_sync(0xffffffffu, s1, o);
+          s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+          s3 += __shfl_xor_sync(0xffffffffu, s3, o);
+        }
         if (x_mine) {
-          dst[threadIdx.x] = quant_vals<QT>(xv, eg == kNoExp ? 0 : -eg);
-          atomicMax(&s_xmax, eg);
+          dst[gi].p1[part] = b1;
+          dst[gi].p2[part] = b2;
+          dst[gi].p3[part] = b3;
+          if (part == 0) {
+            constexpr int off = QT == kQ8 ? 128 : 8;
+            dst[gi].k12 = off * (s1 * 127 + s2);
+            dst[gi].k3 = off * s3;
+            dst[gi].sf = inv > 0.f ? ms / 127.f / 16129.f : 0.f;
+            atomicMax(&s_xmax, eg);
+          }
         }
         named_bar_sync(1, kConsumers * 32);
-        if (x_mine) rescale_group<QT>(dst[threadIdx.x], eg, vector_exponent(s_xmax));
+        if (x_mine && part == 0) rescale_group<QT>(dst[gi], eg, vector_exponent(s_xmax));
         if (threadIdx.x == 0) s_xexp = vector_exponent(s_xmax);
         named_bar_sync(1, kConsumers * 32);
+      } else {
+        split_vectors<QT>(x, cg.n_vec, cg.n_vec, reinterpret_cast<XQ<QT>*>(sm.vq), &s_xmax, &s_xexp);
       }
       XQ<QT> xr[VPL];
 #pragma unroll

@@ -87,6 +87,15 @@ def test_ragged_shapes_decode(qtype, kernels, monkeypatch):
     _decode_run(shape, 4, 40, seed=3)
 
 
+@pytest.mark.parametrize("hidden", [2048, 4096])
+@pytest.mark.parametrize("qtype", [synth.Q8_0, synth.Q4_0])
+def test_fused_decode_x_split_widths(qtype, hidden):
+    """The fused kernel splits x four values per thread where x has at most 512 such words
+    (hidden 2048: every consumer thread one word) and one group per thread above that (hidden
+    4096); both against the oracle."""
+    _decode_run(Shape(1, hidden, 16, 4, 256, qtype, model_seed=12), 6, 12, seed=4)
+
+
 @pytest.mark.parametrize("kernels", ["fused", "pipelined"])
 def test_q4_0_decode_full_width(kernels, monkeypatch):
     """Q4_0 at hidden 2048 / intermediate 768 (the 48-layer Q4_0 shape), one layer, batch 1."""
