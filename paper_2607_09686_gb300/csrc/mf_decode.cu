@@ -726,7 +726,50 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       split_vectors<QT, true>(d.h, f.n_hvec, nvec, reinterpret_cast<XQ<QT>*>(sm.vq), s_hmax, s_hexp);  // other blocks wrote h
       float* red = sm.red + cg.max_mine * kConsumers;  // [k][rpc]
       const int wpe = kConsumers / k, j = warp / wpe, sub = warp % wpe;
-      if (j < mine_d && ok) {
+      if (QT == kQ8 && j < mine_d && ok && nvec > 32 && nvec <= 48) {
+        // rows of at most 48 vectors: half-warp h (lanes 16 h ..) takes row 2 p + h of the warp's
+        // row pairs p = sub, sub + wpe, ..., each lane three vectors: no idle lanes, a 16-lane sum
+        const int hl = lane & 15, half = lane >> 4;
+        XQ<QT> hr3[3];
+#pragma unroll
+        for (int i = 0; i < 3; ++i) {
+          const int v = hl + 16 * i;
+          if (v < nvec) hr3[i] = hq[j * nvec + v];
+        }
+        const int e = s_hexp[j];
+        if ((ok = mbar_wait(&full_d[j], 0, d.wait_ns))) {
+          const unsigned char* st = dbuf + (size_t)j * f.dn_bytes;
+          for (int p0 = sub; 2 * p0 < nrows; p0 += 2 * wpe) {  // two row pairs at a time
+            float acc[2];
+#pragma unroll
+            for (int pp = 0; pp < 2; ++pp) {
+              const int row = 2 * (p0 + pp * wpe) + half;
+              acc[pp] = 0.f;
+              if (row < nrows) {
+                const unsigned char* q = st + (size_t)row * rs;
+                const __half* sc = reinterpret_cast<const __half*>(q + d.lay.o_ds);
+#pragma unroll
+                for (int i = 0; i < 3; ++i) {
+                  const int v = hl + 16 * i;
+                  if (v < nvec)
+                    acc[pp] = fmaf(dot_q<QT>(*reinterpret_cast<const uint4*>(q + 16 * v), hr3[i]),
+                                   __half2float(sc[scale_index<QT>(v)]), acc[pp]);
+                }
+              }
+            }
+#pragma unroll
+            for (int o = 8; o > 0; o >>= 1)
+#pragma unroll
+              for (int pp = 0; pp < 2; ++pp) acc[pp] += __shfl_xor_sync(0xffffffffu, acc[pp], o);
+            if (hl == 0)
+#pragma unroll
+              for (int pp = 0; pp < 2; ++pp) {
+                const int row = 2 * (p0 + pp * wpe) + half;
+                if (row < nrows) red[j * f.rpc + row] = scale2(acc[pp], e);
+              }
+          }
+        }
+      } else if (j < mine_d && ok) {
         XQ<QT> hr[VPLD];
 #pragma unroll
         for (int i = 0; i < VPLD; ++i) {

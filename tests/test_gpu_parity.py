@@ -96,6 +96,13 @@ def test_fused_decode_x_split_widths(qtype, hidden):
     _decode_run(Shape(1, hidden, 16, 4, 256, qtype, model_seed=12), 6, 12, seed=4)
 
 
+@pytest.mark.parametrize("inter", [640, 768])
+def test_fused_decode_half_warp_down_rows(inter):
+    """Q8_0 down rows of 40 and 48 16-byte vectors (inter 640, 768): the fused kernel gives each
+    half-warp a row and each lane three vectors (idle lanes in the 40-vector rows)."""
+    _decode_run(Shape(2, 512, 16, 8, inter, synth.Q8_0, model_seed=13), 9, 10, seed=5)
+
+
 @pytest.mark.parametrize("kernels", ["fused", "pipelined"])
 def test_q4_0_decode_full_width(kernels, monkeypatch):
     """Q4_0 at hidden 2048 / intermediate 768 (the 48-layer Q4_0 shape), one layer, batch 1."""
