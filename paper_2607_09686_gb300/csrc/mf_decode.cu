@@ -421,7 +421,6 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   __shared__ float s_g[kMaxTopK];
   __shared__ int s_miss[kMaxTopK];
   __shared__ int s_gord[kMaxItemsF];  // the block's gate/up items: resident experts' first
-  __shared__ int s_ord[kMaxTopK];     // ranks: resident experts', then missed experts'
   __shared__ int s_nres, s_nb;        // how many of them are resident; ring B's stages
   __shared__ int s_xmax, s_xexp;      // exponent of x's largest magnitude (split scale)
   __shared__ int s_hmax[kMaxTopK], s_hexp[kMaxTopK];  // the same for each expert's h
@@ -469,24 +468,25 @@ __global__ void __launch_bounds__(kThreadsF, 1)
     s_miss[threadIdx.x] = d.umiss[threadIdx.x];
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    // list position p = blockIdx.x + t * gridDim.x; the list holds the resident experts' items,
-    // then the missed experts' (ranks in order within each); item id = rank * (I / R) + row block
+  if (warp == 0) {
+    // list position p = blockIdx.x + t * gridDim.x (lane t); the list holds the resident experts'
+    // items, then the missed experts' (ranks in order within each); item id = rank * (I / R) + row
+    // block.  Position q of the expert list: the q-th resident rank, or the (q - n_res)-th missed one.
     const int nrb = d.I / cg.R;
-    int* ord = s_ord;
-    int n_res_e = 0;
-    for (int j = 0; j < k; ++j)
-      if (!s_miss[j]) ord[n_res_e++] = j;
-    for (int j = 0, n = n_res_e; j < k; ++j)
-      if (s_miss[j]) ord[n++] = j;
-    int nres = 0;
-    for (int t = 0; t < mine_g; ++t) {
-      const int p = (int)blockIdx.x + t * (int)gridDim.x;
-      s_gord[t] = ord[p / nrb] * nrb + p % nrb;
-      nres += p < n_res_e * nrb;
+    const unsigned kmask = (1u << k) - 1u;
+    const unsigned res = __ballot_sync(0xffffffffu, lane < k && !s_miss[lane]);
+    const int n_res_e = __popc(res);
+    for (int t = lane; t < mine_g; t += 32) {
+      const int p = (int)blockIdx.x + t * (int)gridDim.x, q = p / nrb;
+      unsigned m = q < n_res_e ? res : (~res & kmask);
+      for (int c = q < n_res_e ? q : q - n_res_e; c > 0; --c) m &= m - 1u;  // drop the c lowest ranks
+      s_gord[t] = (__ffs(m) - 1) * nrb + p % nrb;
     }
-    s_nres = nres;
-    s_nb = n_res_e < k ? 2 : 0;  // ring B only when the call has a missed expert (NS >= 4)
+    if (lane == 0) {
+      const int lim = n_res_e * nrb - (int)blockIdx.x;  // items t with p < n_res_e * nrb
+      s_nres = lim <= 0 ? 0 : min(mine_g, (lim + (int)gridDim.x - 1) / (int)gridDim.x);
+      s_nb = n_res_e < k ? 2 : 0;  // ring B only when the call has a missed expert (NS >= 4)
+    }
   }
   __syncthreads();
 
