@@ -421,6 +421,7 @@ __global__ void __launch_bounds__(kThreadsF, 1)
   __shared__ float s_g[kMaxTopK];
   __shared__ int s_miss[kMaxTopK];
   __shared__ int s_gord[kMaxItemsF];  // the block's gate/up items: resident experts' first
+  __shared__ const uint8_t* s_gsrc[kMaxItemsF];  // ... their HBM records (resident items)
   __shared__ int s_nres, s_nb;        // how many of them are resident; ring B's stages
   __shared__ int s_xmax, s_xexp;      // exponent of x's largest magnitude (split scale)
   __shared__ int s_hmax[kMaxTopK], s_hexp[kMaxTopK];  // the same for each expert's h
@@ -480,7 +481,9 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       const int p = (int)blockIdx.x + t * (int)gridDim.x, q = p / nrb;
       unsigned m = q < n_res_e ? res : (~res & kmask);
       for (int c = q < n_res_e ? q : q - n_res_e; c > 0; --c) m &= m - 1u;  // drop the c lowest ranks
-      s_gord[t] = (__ffs(m) - 1) * nrb + p % nrb;
+      const int u = __ffs(m) - 1, rb = p % nrb;
+      s_gord[t] = u * nrb + rb;
+      s_gsrc[t] = s_gu[u] + (size_t)rb * cg.R * d.lay.rs_gu;
     }
     if (lane == 0) {
       const int lim = n_res_e * nrb - (int)blockIdx.x;  // items t with p < n_res_e * nrb
@@ -519,10 +522,9 @@ __global__ void __launch_bounds__(kThreadsF, 1)
       for (int t = 0; t < n_issue; ++t, ++it) {
         if (t == first) issue_down_hits();
         if (it >= NA && !(ok = mbar_wait(&sm.empty[ring.s], ring.phase ^ 1u, d.wait_ns))) break;
-        const int item = s_gord[t], u = item / nrb, rb = item % nrb;
         uint64_t* bar = &sm.full[ring.s];
         mbar_arrive_tx(bar, bytes);
-        bulk_g2s_hint(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gu[u] + (size_t)rb * R * rs, bytes, bar, pol);
+        bulk_g2s_hint(sm.stage0 + (size_t)ring.s * f.stage_bytes, s_gsrc[t], bytes, bar, pol);
         ring.next(NA);
       }
       if (ok && !d_issued && !d.hold) issue_down_hits();
