@@ -56,7 +56,7 @@ def workload_name(cache_pct: float = HEAD_PCT, klass: str = HEAD_CLASS) -> str:
 # DRAM bytes (read + write) of one launch of the roofline kernel (the fused one-token FFN) from
 # the ncu capture summarised under profiles/, valid while the kernel sources hash to `sha`
 # (otherwise the line reports null: the counters no longer describe the kernel that ran).
-KERNEL_TRAFFIC = {"sha": "1e4b5f386e62f8d4", "bytes": 40225536,
+KERNEL_TRAFFIC = {"sha": "66dcaba3a9f04fbd", "bytes": 40218368,
                   "files": ("paper_2607_09686_gb300/csrc/mf_decode.cu", "paper_2607_09686_gb300/csrc/mf_dequant.cuh",
                             "paper_2607_09686_gb300/csrc/mf_internal.cuh")}
 
